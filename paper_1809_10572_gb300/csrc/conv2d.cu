@@ -1,0 +1,654 @@
+// conv2d.cu -- bit-precise convolution as an implicit GEMM on the tcgen05
+// tensor cores.
+//
+// The paper's DNN convolution (section 7, Fig. 12, direct-sum2d) is
+//   acc[n][k][ho][wo] = sum_{c,r,s} act[n][c][ho*st-p+r][wo*st-p+s] * wt[k][c][r][s].
+// Here it is the GEMM D[M x K] = A[M x Kg] * B[K x Kg]^T with M = N*Ho*Wo
+// output pixels and a reduction index Kg running over (tap, packed word,
+// lane). The paper's own engine -- 1D convolution by one wide scalar
+// multiply per packed word (section 5) -- is a CPU technique; on GB300 the
+// dense contraction belongs on the tensor cores, and the packing still pays
+// where the data moves: activations and weights stay packed in HBM and in
+// L2, and are widened only in shared memory, right before the MMA (the
+// "unpack to the native type" baseline of section 7, moved on-chip).
+//
+// Exactness. tcgen05 has no integer MMA on sm_103a, so lanes are widened to
+// fp16, which holds every integer of [-128, 255] exactly; products are exact
+// and the fp32 accumulators hold exact integers while every partial sum
+// stays below 2^24. The host only launches shapes whose bound
+// R*S*C*max|a|*max|w| is below 2^24.
+//
+// CTA = 6 warps, one 128-pixel tile x one block of output channels:
+//   warp 0      TMEM allocation; lane 0 streams weight tiles with TMA
+//   warp 1      lane 0 issues tcgen05.mma (128 x N x 16 per instruction)
+//   warps 2-5   load packed activation words (implicit im2col, zero pad),
+//               widen them to fp16 in the 128-byte-swizzled K-major layout,
+//               then run the epilogue: tcgen05.ld of the fp32 accumulators,
+//               int32 store and/or requantize-and-pack to fo.
+// Weights are widened once per call into the workspace (a [K][Kg] fp16
+// matrix in the same Kg order) by wprep_kernel.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_fp16.h>
+
+#include <mutex>
+
+#include "samd_internal.cuh"
+#include "tc_ptx.cuh"
+
+namespace samd {
+
+// Sticky record of a bounded wait that ran out (SAMD_ETIMEOUT), per device.
+__device__ int g_conv_status;
+
+namespace {
+
+constexpr int BM = 128;             // output pixels per tile = MMA M = TMEM lanes
+constexpr int BK = 64;              // fp16 reduction elements per chunk = one 128-byte row
+constexpr int kThreads = 192;
+constexpr int kUnpackThreads = 128;
+constexpr uint32_t kATileBytes = BM * BK * 2;
+constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s
+
+__host__ __device__ constexpr bool pair16(int bits) { return bits == 1 || bits == 2 || bits == 4 || bits == 8; }
+
+// The lane of a packed word held by reduction position `pos` (0 <= pos < L)
+// of that word. For lane widths dividing 16, positions 2p and 2p+1 hold
+// lanes p and p + 16/bits of the same 32-bit half, which sit exactly 16 bits
+// apart, so one masked shift widens both at once. Other widths keep lane
+// order. A and B use the same map, so the dot products are unchanged.
+__host__ __device__ constexpr int kpos_lane(int bits, int pos) {
+  if (pair16(bits)) {
+    int g = 32 / bits, half = pos / g, jj = pos % g;
+    return half * g + jj / 2 + (jj & 1) * (g / 2);
+  }
+  return pos;
+}
+
+struct ConvArgs {
+  const void *act;
+  int32_t *acc_out;
+  void *packed_out;
+  int N, C, H, W, K, R, S, stride, pad, Ho, Wo;
+  long long M;
+  int wpr;          // activation words per pixel
+  int words_total;  // R * S * wpr: reduction length in packed words
+  int nchunks;      // ceil(words_total / words per chunk)
+  int NBc;          // output channels per channel block
+  int n_mma;        // MMA N (NBc rounded up to 16)
+  int stages;
+  uint32_t tmem_cols;
+  int out_bits, out_signed, out_lane_w, out_L, out_word64, out_wpr;
+  int shift;
+};
+
+__device__ __forceinline__ uint32_t hsub2_bits(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+
+// Widening of one 64-position row of the A tile (one pixel, one chunk).
+template <typename W, int BITS, bool SIGNED>
+struct AUnpack {
+  static constexpr int WB = WordTraits<W>::kBits;
+  static constexpr int L = WB / BITS;
+  static constexpr int WC = BK / L;        // packed words per chunk
+  static constexpr int KUSED = WC * L;     // positions holding lanes; the rest are zero
+  static constexpr uint32_t LM = (1u << BITS) - 1;
+  static constexpr uint32_t OFF = SIGNED ? (1u << (BITS - 1)) : 0u;  // offset-binary zero
+  static constexpr uint32_t BIAS = 0x6400u + OFF;                   // fp16 bits of 1024 + OFF
+  static constexpr uint32_t BIAS2 = BIAS | (BIAS << 16);
+
+  static constexpr W sign_mask() {
+    W m = 0;
+    for (int i = 0; i < L; ++i) m |= W(1) << (i * BITS + BITS - 1);
+    return m;
+  }
+
+  template <int POS>
+  __device__ static __forceinline__ uint32_t field(W w) {
+    return static_cast<uint32_t>(w >> (kpos_lane(BITS, POS) * BITS)) & LM;
+  }
+
+  // A lane pattern v (offset binary when signed) becomes fp16 1024 + v by
+  // or-ing it into the mantissa of 1024.0; subtracting 1024 + OFF leaves the
+  // lane's value exactly. A zero word (padding) therefore widens to zeros.
+  template <int P>
+  __device__ static __forceinline__ uint32_t pair(const W (&w)[WC]) {
+    constexpr int j0 = 2 * P, j1 = 2 * P + 1;
+    if constexpr (j0 >= KUSED) {
+      return 0u;
+    } else if constexpr (pair16(BITS)) {
+      constexpr int q = j0 / L, pos = j0 % L, g = 32 / BITS, half = pos / g;
+      constexpr int lane0 = kpos_lane(BITS, pos) - half * g;
+      const uint32_t x = static_cast<uint32_t>(w[q] >> (half * 32));
+      const uint32_t t = ((x >> (lane0 * BITS)) & (LM | (LM << 16))) | 0x64006400u;
+      return hsub2_bits(t, BIAS2);
+    } else {
+      const uint32_t v0 = field<j0 % L>(w[j0 / L]);
+      uint32_t v1 = OFF;
+      if constexpr (j1 < KUSED) v1 = field<j1 % L>(w[j1 / L]);
+      return hsub2_bits(v0 | (v1 << 16) | 0x64006400u, BIAS2);
+    }
+  }
+
+  template <int... P>
+  __device__ static __forceinline__ void pairs(const W (&w)[WC], uint32_t (&h)[32],
+                                               std::integer_sequence<int, P...>) {
+    ((h[P] = pair<P>(w)), ...);
+  }
+
+  // Widen one pixel's chunk and store it as row `row` of a 128-byte
+  // swizzled K-major tile: 16-byte block c goes to block c ^ (row % 8).
+  __device__ static __forceinline__ void unpack_row(W (&w)[WC], uint8_t *tile, int row) {
+    if constexpr (SIGNED) {
+#pragma unroll
+      for (int q = 0; q < WC; ++q) w[q] ^= sign_mask();
+    }
+    uint32_t h[32];
+    pairs(w, h, std::make_integer_sequence<int, 32>{});
+    uint8_t *rp = tile + row * 128;
+    const int swz = row & 7;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      *reinterpret_cast<uint4 *>(rp + ((c ^ swz) << 4)) = make_uint4(h[4 * c], h[4 * c + 1], h[4 * c + 2], h[4 * c + 3]);
+    }
+  }
+};
+
+// Gathers the packed words of one pixel's chunk: word kw of the reduction is
+// word (kw mod wpr) of the input pixel at tap kw / wpr; taps outside the
+// image and words past the end read zero.
+template <typename W, int WC>
+struct AGather {
+  const W *act;
+  int H, W_, wpr, S, stride, pad, words_total;
+  int n, oh, ow;
+  bool row_valid;
+
+  __device__ __forceinline__ const W *pixel(int tap, bool &valid) const {
+    int r = tap / S, s = tap - (tap / S) * S;
+    int ih = oh * stride - pad + r, iw = ow * stride - pad + s;
+    valid = row_valid && ih >= 0 && ih < H && iw >= 0 && iw < W_;
+    return act + ((static_cast<long long>(n) * H + ih) * W_ + iw) * wpr;
+  }
+
+  __device__ __forceinline__ void load(int chunk, W (&dst)[WC]) const {
+    const int kw0 = chunk * WC;
+    int tap = kw0 / wpr, wi = kw0 - tap * wpr;
+    bool valid;
+    const W *px = pixel(tap, valid);
+#pragma unroll
+    for (int q = 0; q < WC; ++q) {
+      dst[q] = (valid && kw0 + q < words_total) ? __ldg(px + wi) : W(0);
+      if (++wi == wpr) {
+        wi = 0;
+        ++tap;
+        px = pixel(tap, valid);
+      }
+    }
+  }
+};
+
+template <typename W, int BITS, bool SIGNED>
+__global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_b,
+                                                               const ConvArgs args) {
+  using U = AUnpack<W, BITS, SIGNED>;
+  constexpr int WC = U::WC;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ int s_skip;
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int ST = args.stages;
+  const uint32_t b_bytes = static_cast<uint32_t>(args.n_mma) * 128u;
+  uint8_t *sA = smem;
+  uint8_t *sB = smem + ST * kATileBytes;
+  uint64_t *bars = reinterpret_cast<uint64_t *>(sB + ST * b_bytes);
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 3 * ST + 2);
+  auto full_a = [&](int s) { return ptx::smem_addr(bars + s); };
+  auto full_b = [&](int s) { return ptx::smem_addr(bars + ST + s); };
+  auto empty = [&](int s) { return ptx::smem_addr(bars + 2 * ST + s); };
+  const uint32_t acc_bar = ptx::smem_addr(bars + 3 * ST);
+  const uint32_t drain_bar = ptx::smem_addr(bars + 3 * ST + 1);
+
+  volatile int *status = &g_conv_status;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) s_skip = *status;  // an earlier failure: leave the outputs alone
+  __syncthreads();
+  if (s_skip) return;
+
+  if (warp == 0) {
+    ptx::tmem_alloc(ptx::smem_addr(tmem_holder), args.tmem_cols);
+    ptx::tmem_relinquish();
+  }
+  if (threadIdx.x == 32) {
+    for (int s = 0; s < ST; ++s) {
+      ptx::mbar_init(full_a(s), kUnpackThreads);
+      ptx::mbar_init(full_b(s), 1);
+      ptx::mbar_init(empty(s), 1);
+    }
+    ptx::mbar_init(acc_bar, 1);
+    ptx::mbar_init(drain_bar, 1);
+    ptx::fence_barrier_init();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  const int nb = blockIdx.y;
+  bool ok = true;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---- weight tiles by TMA ----
+      ptx::prefetch_tmap(&tmap_b);
+      int issued = 0;
+      for (int c = 0; c < args.nchunks; ++c) {
+        const int s = c % ST, round = c / ST;
+        if (round > 0 && !ptx::mbar_wait_bounded(empty(s), (round - 1) & 1, status, kWaitLimitNs)) {
+          ok = false;
+          break;
+        }
+        ptx::mbar_arrive_expect_tx(full_b(s), b_bytes);
+        ptx::tma_load_2d(ptx::smem_addr(sB + s * b_bytes), &tmap_b, c * BK, nb * args.n_mma, full_b(s));
+        issued = c + 1;
+      }
+      if (!ok) {
+        // do not leave copies in flight into shared memory: wait (bounded) for
+        // the ones whose completion nobody observed
+        for (int c = issued - ST < 0 ? 0 : issued - ST; c < issued; ++c)
+          ptx::mbar_wait_bounded(full_b(c % ST), (c / ST) & 1, status, kWaitLimitNs / 10);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---- MMA issue ----
+      const uint32_t idesc = ptx::idesc_f16_f32(BM, args.n_mma);
+      for (int c = 0; c < args.nchunks; ++c) {
+        const int s = c % ST, round = c / ST;
+        if (!ptx::mbar_wait_bounded(full_a(s), round & 1, status, kWaitLimitNs) ||
+            !ptx::mbar_wait_bounded(full_b(s), round & 1, status, kWaitLimitNs)) {
+          ok = false;
+          break;
+        }
+        ptx::tc_fence_after();
+        const uint64_t adesc = ptx::sw128_kmajor_desc(ptx::smem_addr(sA + s * kATileBytes));
+        const uint64_t bdesc = ptx::sw128_kmajor_desc(ptx::smem_addr(sB + s * b_bytes));
+        int words = args.words_total - c * WC;
+        if (words > WC) words = WC;
+        const int ksteps = (words * U::L + 15) / 16;
+        for (int kk = 0; kk < ksteps; ++kk)
+          ptx::mma_f16(tmem_base, adesc + 2 * kk, bdesc + 2 * kk, idesc, (c > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma_commit(empty(s));
+      }
+      if (ok) ptx::mma_commit(acc_bar);
+      // all MMAs of this CTA must be complete before TMEM is released
+      ptx::mma_commit(drain_bar);
+      int quiet = 0;
+      ptx::mbar_wait_bounded(drain_bar, 0, &quiet, kWaitLimitNs);
+    }
+  } else {
+    // ---- activation gather + widen, then the epilogue ----
+    const int quad = warp & 3;  // TMEM lanes 32*quad .. 32*quad+31 belong to this warp
+    const int row = quad * 32 + lane;
+    const long long m = static_cast<long long>(blockIdx.x) * BM + row;
+    AGather<W, WC> g;
+    g.act = static_cast<const W *>(args.act);
+    g.H = args.H;
+    g.W_ = args.W;
+    g.wpr = args.wpr;
+    g.S = args.S;
+    g.stride = args.stride;
+    g.pad = args.pad;
+    g.words_total = args.words_total;
+    g.row_valid = m < args.M;
+    {
+      const long long mm = g.row_valid ? m : 0;
+      g.ow = static_cast<int>(mm % args.Wo);
+      const long long t = mm / args.Wo;
+      g.oh = static_cast<int>(t % args.Ho);
+      g.n = static_cast<int>(t / args.Ho);
+    }
+    W cur[WC], nxt[WC];
+    g.load(0, cur);
+    for (int c = 0; c < args.nchunks; ++c) {
+      if (c + 1 < args.nchunks) g.load(c + 1, nxt);
+      const int s = c % ST, round = c / ST;
+      if (round > 0 && !ptx::mbar_wait_bounded(empty(s), (round - 1) & 1, status, kWaitLimitNs)) {
+        ok = false;
+        break;
+      }
+      U::unpack_row(cur, sA + s * kATileBytes, row);
+      ptx::fence_proxy_async_smem();
+      ptx::mbar_arrive(full_a(s));
+#pragma unroll
+      for (int q = 0; q < WC; ++q) cur[q] = nxt[q];
+    }
+
+    if (ok) ok = ptx::mbar_wait_bounded(acc_bar, 0, status, kWaitLimitNs);
+    // every thread of the warp must take part in tcgen05.ld
+    ok = __all_sync(0xffffffffu, ok);
+    if (ok) {
+      ptx::tc_fence_after();
+      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16);
+      const int ch0 = nb * args.NBc;
+      const int nvalid = args.K - ch0 < args.NBc ? args.K - ch0 : args.NBc;
+      const bool vec_ok = (args.K % 4 == 0) && (ch0 % 4 == 0);
+      const int lo = lane_lo(args.out_bits, args.out_signed), hi = lane_hi(args.out_bits, args.out_signed);
+      const uint32_t omask = (1u << args.out_bits) - 1;
+      uint64_t wacc = 0;
+      int wl = 0;
+      long long widx = g.row_valid && args.packed_out ? m * args.out_wpr + ch0 / args.out_L : 0;
+      for (int col = 0; col < nvalid; col += 32) {
+        uint32_t r[32];
+        ptx::tmem_ld_32x32b_x32(taddr + col, r);
+        ptx::tmem_wait_ld();
+        if (!g.row_valid) continue;
+        const int cnt = nvalid - col < 32 ? nvalid - col : 32;
+        int v[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = __float2int_rn(__uint_as_float(r[i]));
+        if (args.acc_out) {
+          int32_t *dst = args.acc_out + m * args.K + ch0 + col;
+          if (cnt == 32 && vec_ok) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+              reinterpret_cast<int4 *>(dst)[i] = make_int4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+          } else {
+            for (int i = 0; i < cnt; ++i) dst[i] = v[i];
+          }
+        }
+        if (args.packed_out) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            if (i < cnt) {
+              const int y = clamp_int(v[i] >> args.shift, lo, hi);
+              wacc |= static_cast<uint64_t>(static_cast<uint32_t>(y) & omask) << (wl * args.out_lane_w);
+              if (++wl == args.out_L) {
+                if (args.out_word64)
+                  static_cast<uint64_t *>(args.packed_out)[widx] = wacc;
+                else
+                  static_cast<uint32_t *>(args.packed_out)[widx] = static_cast<uint32_t>(wacc);
+                ++widx;
+                wacc = 0;
+                wl = 0;
+              }
+            }
+          }
+        }
+      }
+      if (g.row_valid && args.packed_out && wl > 0) {
+        if (args.out_word64)
+          static_cast<uint64_t *>(args.packed_out)[widx] = wacc;
+        else
+          static_cast<uint32_t *>(args.packed_out)[widx] = static_cast<uint32_t>(wacc);
+      }
+    }
+  }
+
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem_base, args.tmem_cols);
+  }
+  if (!ok) atomicOr(const_cast<int *>(status), static_cast<int>(SAMD_ETIMEOUT));
+}
+
+// ---- weight widening into the workspace ----------------------------------
+
+struct WPrepArgs {
+  int K, C, RS;
+  int bits_w, signed_w, lane_w_w, Lw, wpr_w;  // weight format
+  int bits_a, La, WC, wpr_a, words_total;      // reduction order set by the activation format
+  int Kpad, n_mma, NBc;
+  long long rows_total;
+};
+
+template <typename WW>
+__global__ void __launch_bounds__(256) wprep_kernel(const WW *__restrict__ wt, __half *__restrict__ B,
+                                                    const WPrepArgs a) {
+  const long long total = a.rows_total * a.Kpad;
+  const uint32_t mask = (1u << a.bits_w) - 1;
+  for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
+       idx += (long long)gridDim.x * blockDim.x) {
+    const long long rowi = idx / a.Kpad;
+    const int kpos = static_cast<int>(idx - rowi * a.Kpad);
+    const int nb = static_cast<int>(rowi / a.n_mma), r = static_cast<int>(rowi % a.n_mma);
+    const int k = nb * a.NBc + r;
+    const int chunk = kpos / BK, j = kpos % BK;
+    const int q = j / a.La, pos = j % a.La;
+    int v = 0;
+    if (r < a.NBc && k < a.K && q < a.WC) {
+      const int kw = chunk * a.WC + q;
+      if (kw < a.words_total) {
+        const int tap = kw / a.wpr_a, wi = kw % a.wpr_a;
+        const int ch = wi * a.La + kpos_lane(a.bits_a, pos);
+        if (ch < a.C) {
+          const long long wrow = static_cast<long long>(k) * a.RS + tap;
+          const WW word = wt[wrow * a.wpr_w + ch / a.Lw];
+          const uint32_t p = static_cast<uint32_t>(word >> ((ch % a.Lw) * a.lane_w_w)) & mask;
+          v = lane_value(p, a.bits_w, a.signed_w);
+        }
+      }
+    }
+    B[idx] = __int2half_rn(v);
+  }
+}
+
+// ---- host side -------------------------------------------------------------
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_tiled() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+struct Plan {
+  int wpr, words_total, La, WC, nchunks, Kpad, NBc, n_mma, nblocks, stages, Ho, Wo;
+  long long M;
+  uint32_t tmem_cols;
+  size_t smem_bytes;
+  size_t ws_bytes;
+};
+
+int lanes_of(samd_fmt f) { return lanes_per_word(f); }
+
+bool make_plan(const samd_conv_desc *d, samd_fmt fa, const samd_fmt *fo_or_null, Plan &p) {
+  p.La = lanes_of(fa);
+  if (p.La == 0) return false;
+  p.WC = BK / p.La;
+  p.wpr = static_cast<int>((d->C + p.La - 1) / p.La);
+  p.words_total = d->R * d->S * p.wpr;
+  p.nchunks = (p.words_total + p.WC - 1) / p.WC;
+  p.Kpad = p.nchunks * BK;
+  p.Ho = (d->H + 2 * d->pad - d->R) / d->stride + 1;
+  p.Wo = (d->W + 2 * d->pad - d->S) / d->stride + 1;
+  p.M = static_cast<long long>(d->N) * p.Ho * p.Wo;
+  if (d->K <= 256) {
+    p.NBc = d->K;
+  } else {
+    int Lo = fo_or_null ? lanes_of(*fo_or_null) : 1;
+    p.NBc = (256 / Lo) * Lo;
+  }
+  p.n_mma = (p.NBc + 15) / 16 * 16;
+  p.nblocks = (d->K + p.NBc - 1) / p.NBc;
+  uint32_t cols = 32;
+  while (cols < static_cast<uint32_t>(p.n_mma)) cols <<= 1;
+  p.tmem_cols = cols;
+  const size_t stage_bytes = kATileBytes + static_cast<size_t>(p.n_mma) * 128;
+  int st = static_cast<int>((100 * 1024) / stage_bytes);
+  if (st < 2) st = 2;
+  if (st > 6) st = 6;
+  p.stages = st;
+  p.smem_bytes = 1024 + st * stage_bytes + (3 * st + 2) * 8 + 16;
+  p.ws_bytes = static_cast<size_t>(p.nblocks) * p.n_mma * p.Kpad * sizeof(__half);
+  return true;
+}
+
+template <typename W, int BITS, bool SIGNED>
+cudaError_t launch_conv_variant(const CUtensorMap &tmap, const ConvArgs &args, dim3 grid, size_t smem,
+                                cudaStream_t s) {
+  auto kern = conv_tc_kernel<W, BITS, SIGNED>;
+  // the attribute is per function and device; setting it again is harmless
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  kern<<<grid, kThreads, smem, s>>>(tmap, args);
+  return cudaGetLastError();
+}
+
+template <typename W>
+cudaError_t launch_conv_word(samd_fmt fa, const CUtensorMap &tmap, const ConvArgs &args, dim3 grid, size_t smem,
+                             cudaStream_t s) {
+  switch (fa.bits * 2 + (fa.is_signed ? 1 : 0)) {
+#define SAMD_CONV_CASE(B)                                                              \
+  case 2 * B:                                                                          \
+    return launch_conv_variant<W, B, false>(tmap, args, grid, smem, s);                \
+  case 2 * B + 1:                                                                      \
+    return launch_conv_variant<W, B, true>(tmap, args, grid, smem, s);
+    SAMD_CONV_CASE(1) SAMD_CONV_CASE(2) SAMD_CONV_CASE(3) SAMD_CONV_CASE(4)
+    SAMD_CONV_CASE(5) SAMD_CONV_CASE(6) SAMD_CONV_CASE(7) SAMD_CONV_CASE(8)
+#undef SAMD_CONV_CASE
+    default:
+      return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace
+
+size_t conv2d_workspace_size(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw) {
+  (void)fw;
+  Plan p;
+  if (!make_plan(d, fa, nullptr, p)) return 0;
+  // the channel blocking depends on the output format only above 256
+  // channels; reserve the largest layout (one lane per word block)
+  if (d->K > 256) {
+    Plan q = p;
+    q.NBc = 250;  // smallest block any output format yields (10 lanes per word)
+    q.n_mma = 256;
+    q.nblocks = (d->K + q.NBc - 1) / q.NBc;
+    size_t big = static_cast<size_t>(q.nblocks) * q.n_mma * q.Kpad * sizeof(__half);
+    return big > p.ws_bytes ? big : p.ws_bytes;
+  }
+  return p.ws_bytes;
+}
+
+samd_status conv2d_nhwc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
+                        int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, void *workspace,
+                        size_t workspace_bytes, cudaStream_t s) {
+  Plan p;
+  if (!make_plan(d, fa, packed_out ? &fo : nullptr, p)) return SAMD_EINVAL;
+  if (workspace_bytes < p.ws_bytes) return SAMD_ESHAPE;
+  if (p.M == 0) return SAMD_OK;
+  EncodeTiledFn enc = encode_tiled();
+  if (!enc) return SAMD_ECUDA;
+
+  // 1. widen the weights into the reduction order of the activations
+  WPrepArgs wa;
+  wa.K = d->K;
+  wa.C = d->C;
+  wa.RS = d->R * d->S;
+  wa.bits_w = fw.bits;
+  wa.signed_w = fw.is_signed;
+  wa.lane_w_w = fw.bits + fw.spacer;
+  wa.Lw = lanes_per_word(fw);
+  wa.wpr_w = static_cast<int>(words_per_row(fw, d->C));
+  wa.bits_a = fa.bits;
+  wa.La = p.La;
+  wa.WC = p.WC;
+  wa.wpr_a = p.wpr;
+  wa.words_total = p.words_total;
+  wa.Kpad = p.Kpad;
+  wa.n_mma = p.n_mma;
+  wa.NBc = p.NBc;
+  wa.rows_total = static_cast<long long>(p.nblocks) * p.n_mma;
+  __half *B = static_cast<__half *>(workspace);
+  {
+    const long long total = wa.rows_total * wa.Kpad;
+    const int grid = grid_for(total, 256, sm_count() * 8);
+    if (fw.word_bits == 32)
+      wprep_kernel<uint32_t><<<grid, 256, 0, s>>>(static_cast<const uint32_t *>(wt), B, wa);
+    else
+      wprep_kernel<uint64_t><<<grid, 256, 0, s>>>(static_cast<const uint64_t *>(wt), B, wa);
+    if (cudaGetLastError() != cudaSuccess) return SAMD_ECUDA;
+  }
+
+  // 2. tensor map over the widened weights: [rows_total][Kpad] fp16, tiles of
+  //    n_mma rows x 64 elements, 128-byte swizzle
+  CUtensorMap tmap;
+  cuuint64_t gdim[2] = {static_cast<cuuint64_t>(p.Kpad), static_cast<cuuint64_t>(wa.rows_total)};
+  cuuint64_t gstride[1] = {static_cast<cuuint64_t>(p.Kpad) * sizeof(__half)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(p.n_mma)};
+  cuuint32_t estride[2] = {1, 1};
+  CUresult cr = enc(&tmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, workspace, gdim, gstride, box, estride,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (cr != CUDA_SUCCESS) return SAMD_ECUDA;
+
+  // 3. the convolution
+  ConvArgs a;
+  a.act = act;
+  a.acc_out = acc_out;
+  a.packed_out = packed_out;
+  a.N = d->N;
+  a.C = d->C;
+  a.H = d->H;
+  a.W = d->W;
+  a.K = d->K;
+  a.R = d->R;
+  a.S = d->S;
+  a.stride = d->stride;
+  a.pad = d->pad;
+  a.Ho = p.Ho;
+  a.Wo = p.Wo;
+  a.M = p.M;
+  a.wpr = p.wpr;
+  a.words_total = p.words_total;
+  a.nchunks = p.nchunks;
+  a.NBc = p.NBc;
+  a.n_mma = p.n_mma;
+  a.stages = p.stages;
+  a.tmem_cols = p.tmem_cols;
+  a.out_bits = packed_out ? fo.bits : 8;
+  a.out_signed = packed_out ? fo.is_signed : 1;
+  a.out_lane_w = packed_out ? fo.bits + fo.spacer : 8;
+  a.out_L = packed_out ? lanes_per_word(fo) : 1;
+  a.out_word64 = packed_out ? (fo.word_bits == 64) : 0;
+  a.out_wpr = packed_out ? static_cast<int>(words_per_row(fo, d->K)) : 0;
+  a.shift = shift;
+  dim3 grid(static_cast<unsigned>((p.M + BM - 1) / BM), static_cast<unsigned>(p.nblocks));
+  cudaError_t e = fa.word_bits == 32 ? launch_conv_word<uint32_t>(fa, tmap, a, grid, p.smem_bytes, s)
+                                     : launch_conv_word<uint64_t>(fa, tmap, a, grid, p.smem_bytes, s);
+  return e == cudaSuccess ? SAMD_OK : SAMD_ECUDA;
+}
+
+cudaError_t read_device_status(int *status, int reset, cudaStream_t s) {
+  int v = 0;
+  cudaError_t e = cudaMemcpyFromSymbolAsync(&v, g_conv_status, sizeof(int), 0, cudaMemcpyDeviceToHost, s);
+  if (e != cudaSuccess) return e;
+  e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return e;
+  *status = v;
+  if (reset && v != 0) {
+    int zero = 0;
+    e = cudaMemcpyToSymbolAsync(g_conv_status, &zero, sizeof(int), 0, cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  }
+  return e;
+}
+
+}  // namespace samd

@@ -1,0 +1,325 @@
+// elementwise.cu -- lane-wise ops on packed words.
+//
+// Spacer-free formats with the same input and output format take the
+// word-level (SAMD) forms: every lane of a word is updated by a handful of
+// whole-word integer instructions, the way section 3 of the paper adds and
+// subtracts with temporary spacer bits (Fig. 5) and multiplies by masked
+// shift-and-add (Fig. 6). On GB300 this keeps the per-word ALU cost below
+// what HBM bandwidth leaves per word even at 1-2 bit lanes, where a
+// lane-by-lane loop would run 16-32 iterations per word. Words move with
+// 128-bit loads and stores.
+//
+// Everything else (spacer bits, saturating multiply of wide lanes,
+// requantize into another format) takes the per-lane path: one thread per
+// output word, bit-field extract, integer op, clamp or wrap, insert.
+#include "samd_internal.cuh"
+
+namespace samd {
+namespace {
+
+constexpr int kThreads = 256;
+
+// ---- compile-time lane masks for spacer-free lanes -------------------------
+
+template <typename W, int BITS>
+struct Masks {
+  static constexpr int L = WordTraits<W>::kBits / BITS;
+  static constexpr W lsb() {
+    W m = 0;
+    for (int i = 0; i < L; ++i) m |= W(1) << (i * BITS);
+    return m;
+  }
+  static constexpr W kLsb = lsb();                     // bit 0 of every lane
+  static constexpr W kMsb = kLsb << (BITS - 1);        // top bit of every lane
+  static constexpr W kLane = (W(1) << BITS) - 1;       // one lane's bits
+  static constexpr W kLive = kLsb * kLane;             // every lane bit
+};
+
+// Spread a mask holding only lane MSBs over the whole of those lanes.
+template <typename W, int BITS>
+__device__ __forceinline__ W expand_msb(W m) {
+  return (m - (m >> (BITS - 1))) | m;
+}
+
+// Section 3, Fig. 5: add with the lane MSBs as temporary spacers.
+template <typename W, int BITS>
+__device__ __forceinline__ W swar_add(W a, W b) {
+  constexpr W M = Masks<W, BITS>::kMsb;
+  return ((a ^ b) & M) ^ ((a & ~M) + (b & ~M));
+}
+
+// Section 3, Fig. 5: subtract; the minuend's MSBs are set and the
+// subtrahend's cleared so no lane borrows from the next.
+template <typename W, int BITS>
+__device__ __forceinline__ W swar_sub(W a, W b) {
+  constexpr W M = Masks<W, BITS>::kMsb;
+  return ((a ^ b) & M) ^ ((a | M) - (b & ~M)) ^ M;
+}
+
+// Saturating add/sub: detect each lane's overflow from the MSBs of the
+// operands and the wrapped result, then replace those lanes by the bound.
+template <typename W, int BITS>
+__device__ __forceinline__ W swar_add_sat(W a, W b, bool is_signed) {
+  constexpr W M = Masks<W, BITS>::kMsb;
+  constexpr W LIVE = Masks<W, BITS>::kLive;
+  W s = swar_add<W, BITS>(a, b);
+  if (!is_signed) {
+    W carry = ((a & b) | ((a | b) & ~s)) & M;  // carry out of each lane
+    return s | expand_msb<W, BITS>(carry);
+  }
+  W ovf = ~(a ^ b) & (a ^ s) & M;  // same-sign operands, other-sign result
+  W E = expand_msb<W, BITS>(ovf);
+  W na = a & M;
+  W sat = (E & ~expand_msb<W, BITS>(na) & ~M & LIVE) | (E & na);  // 011..1 or 100..0
+  return (s & ~E) | sat;
+}
+
+template <typename W, int BITS>
+__device__ __forceinline__ W swar_sub_sat(W a, W b, bool is_signed) {
+  constexpr W M = Masks<W, BITS>::kMsb;
+  constexpr W LIVE = Masks<W, BITS>::kLive;
+  W d = swar_sub<W, BITS>(a, b);
+  if (!is_signed) {
+    W borrow = ((~a & b) | ((~a | b) & d)) & M;  // borrow out of each lane
+    return d & ~expand_msb<W, BITS>(borrow);
+  }
+  W ovf = (a ^ b) & (a ^ d) & M;  // other-sign operands, result sign differs from a
+  W E = expand_msb<W, BITS>(ovf);
+  W na = a & M;
+  W sat = (E & ~expand_msb<W, BITS>(na) & ~M & LIVE) | (E & na);
+  return (d & ~E) | sat;
+}
+
+// Section 3, Fig. 6: lane-wise multiply, low bits, by masked shift-and-add;
+// in step j the j-th bit of each lane of b selects a << j, cut at the top of
+// the lane by a mask built in one subtraction.
+template <typename W, int BITS>
+__device__ __forceinline__ W swar_mul(W a, W b) {
+  constexpr W LSB = Masks<W, BITS>::kLsb;
+  W acc = 0;
+#pragma unroll
+  for (int j = 0; j < BITS; ++j) {
+    W bit = b & (LSB << j);
+    W write = (bit << (BITS - j)) - bit;
+    acc = swar_add<W, BITS>(acc, (a << j) & write);
+  }
+  return acc;
+}
+
+// Lane-by-lane multiply (cheaper than shift-and-add from 3-bit lanes up).
+template <typename W, int BITS>
+__device__ __forceinline__ W lane_mul(W a, W b, bool is_signed, bool sat) {
+  constexpr int L = Masks<W, BITS>::L;
+  constexpr uint32_t LM = (1u << BITS) - 1;
+  const int lo = lane_lo(BITS, is_signed), hi = lane_hi(BITS, is_signed);
+  W r = 0;
+#pragma unroll
+  for (int i = 0; i < L; ++i) {
+    uint32_t pa = static_cast<uint32_t>(a >> (i * BITS)) & LM;
+    uint32_t pb = static_cast<uint32_t>(b >> (i * BITS)) & LM;
+    uint32_t p;
+    if (sat) {
+      int v = lane_value(pa, BITS, is_signed) * lane_value(pb, BITS, is_signed);
+      p = static_cast<uint32_t>(clamp_int(v, lo, hi)) & LM;
+    } else {
+      p = (pa * pb) & LM;  // low bits are the same for signed and unsigned (section 4.1)
+    }
+    r |= W(p) << (i * BITS);
+  }
+  return r;
+}
+
+template <typename W, int BITS>
+__device__ __forceinline__ W swar_relu(W a, bool is_signed) {
+  if (!is_signed) return a;
+  constexpr W M = Masks<W, BITS>::kMsb;
+  return a & ~expand_msb<W, BITS>(a & M);
+}
+
+// Requantize within the format: floor(x / 2^shift) per lane. A right shift
+// never leaves the lane range, so no clamp is needed. `keep` holds the low
+// (BITS - shift) bits of every lane.
+template <typename W, int BITS>
+__device__ __forceinline__ W swar_shift(W a, int shift, W keep, bool is_signed) {
+  if (shift == 0) return a;
+  W r = (a >> shift) & keep;
+  if (is_signed) {
+    constexpr W M = Masks<W, BITS>::kMsb;
+    W sg = a & M;
+    W t = sg >> (shift - 1);
+    r |= (sg - t) | sg;  // sign fill of the top `shift` bits of negative lanes
+  }
+  return r;
+}
+
+template <typename W, int BITS, int OP>
+__device__ __forceinline__ W apply_op(W a, W b, bool is_signed, bool sat, int shift, W keep) {
+  if constexpr (OP == SAMD_ADD) {
+    return sat ? swar_add_sat<W, BITS>(a, b, is_signed) : swar_add<W, BITS>(a, b);
+  } else if constexpr (OP == SAMD_SUB) {
+    return sat ? swar_sub_sat<W, BITS>(a, b, is_signed) : swar_sub<W, BITS>(a, b);
+  } else if constexpr (OP == SAMD_MUL) {
+    if constexpr (BITS == 1) {
+      if (!sat || !is_signed) return a & b;  // 1-bit: product = AND (u1 never overflows)
+      return lane_mul<W, BITS>(a, b, is_signed, sat);
+    } else if constexpr (BITS == 2) {
+      if (!sat) return swar_mul<W, BITS>(a, b);
+      return lane_mul<W, BITS>(a, b, is_signed, sat);
+    } else {
+      return lane_mul<W, BITS>(a, b, is_signed, sat);
+    }
+  } else if constexpr (OP == SAMD_RELU) {
+    return swar_relu<W, BITS>(a, is_signed);
+  } else {
+    return swar_shift<W, BITS>(a, shift, keep, is_signed);
+  }
+}
+
+template <typename W>
+struct Vec4 {
+  static constexpr int kWords = 16 / sizeof(W);
+};
+
+template <typename W, int BITS, int OP>
+__global__ void __launch_bounds__(kThreads)
+    ew_swar_kernel(const W *__restrict__ a, const W *__restrict__ b, W *__restrict__ out, int64_t nwords,
+                   int is_signed, int sat, int shift) {
+  constexpr int V = Vec4<W>::kWords;
+  constexpr bool kBinary = (OP == SAMD_ADD || OP == SAMD_SUB || OP == SAMD_MUL);
+  W keep = 0;
+  if (OP == SAMD_REQUANT) {
+    int s = shift < BITS ? shift : BITS;
+    keep = Masks<W, BITS>::kLsb * ((W(1) << (BITS - s)) - 1);
+    shift = s;
+  }
+  const int64_t nvec = nwords / V;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < nvec; v += stride) {
+    uint4 ra = __ldcs(reinterpret_cast<const uint4 *>(a) + v);
+    uint4 rb = ra;
+    if (kBinary) rb = __ldcs(reinterpret_cast<const uint4 *>(b) + v);
+    W wa[V], wb[V], wo[V];
+    memcpy(wa, &ra, 16);
+    memcpy(wb, &rb, 16);
+#pragma unroll
+    for (int k = 0; k < V; ++k) wo[k] = apply_op<W, BITS, OP>(wa[k], wb[k], is_signed, sat, shift, keep);
+    uint4 ro;
+    memcpy(&ro, wo, 16);
+    __stcs(reinterpret_cast<uint4 *>(out) + v, ro);
+  }
+  // tail words that do not fill a 128-bit vector
+  for (int64_t w = nvec * V + blockIdx.x * (int64_t)blockDim.x + threadIdx.x; w < nwords; w += stride) {
+    W x = a[w];
+    W y = kBinary ? b[w] : x;
+    out[w] = apply_op<W, BITS, OP>(x, y, is_signed, sat, shift, keep);
+  }
+}
+
+// Per-lane path: any spacer, any output format. One thread per output word.
+struct LaneFmt {
+  int bits, is_signed, lane_w, L;
+};
+
+template <typename WI, typename WO>
+__global__ void __launch_bounds__(kThreads)
+    ew_lane_kernel(int op, LaneFmt fa, const WI *__restrict__ a, const WI *__restrict__ b, LaneFmt fo,
+                   WO *__restrict__ out, int64_t n, int64_t nwords_out, int shift, int sat) {
+  const uint32_t ma = (1u << fa.bits) - 1, mo = (1u << fo.bits) - 1;
+  const int lo = lane_lo(fo.bits, fo.is_signed), hi = lane_hi(fo.bits, fo.is_signed);
+  for (int64_t w = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; w < nwords_out;
+       w += (int64_t)gridDim.x * blockDim.x) {
+    WO word = 0;
+    for (int l = 0; l < fo.L; ++l) {
+      int64_t e = w * fo.L + l;
+      if (e >= n) break;
+      int64_t wi = e / fa.L;
+      int li = static_cast<int>(e - wi * fa.L);
+      int x = lane_value(static_cast<uint32_t>(a[wi] >> (li * fa.lane_w)) & ma, fa.bits, fa.is_signed);
+      int y = 0;
+      if (op == SAMD_ADD || op == SAMD_SUB || op == SAMD_MUL)
+        y = lane_value(static_cast<uint32_t>(b[wi] >> (li * fa.lane_w)) & ma, fa.bits, fa.is_signed);
+      int v;
+      switch (op) {
+        case SAMD_ADD: v = x + y; break;
+        case SAMD_SUB: v = x - y; break;
+        case SAMD_MUL: v = x * y; break;
+        case SAMD_RELU: v = x < 0 ? 0 : x; break;
+        default: v = x >> shift; break;  // arithmetic shift: floor(x / 2^shift)
+      }
+      if (op == SAMD_REQUANT || sat) v = clamp_int(v, lo, hi);
+      word |= WO(static_cast<uint32_t>(v) & mo) << (l * fo.lane_w);
+    }
+    out[w] = word;
+  }
+}
+
+template <typename W, int OP>
+cudaError_t swar_dispatch_bits(int bits, const void *a, const void *b, void *out, int64_t nwords, int is_signed,
+                               int sat, int shift, cudaStream_t s) {
+  int64_t work = nwords / Vec4<W>::kWords + 1;
+  int grid = grid_for(work, kThreads, sm_count() * 8);
+  const W *pa = static_cast<const W *>(a);
+  const W *pb = static_cast<const W *>(b);
+  W *po = static_cast<W *>(out);
+  switch (bits) {
+#define SAMD_EW_CASE(B) \
+  case B:               \
+    ew_swar_kernel<W, B, OP><<<grid, kThreads, 0, s>>>(pa, pb, po, nwords, is_signed, sat, shift); \
+    break;
+    SAMD_EW_CASE(1) SAMD_EW_CASE(2) SAMD_EW_CASE(3) SAMD_EW_CASE(4)
+    SAMD_EW_CASE(5) SAMD_EW_CASE(6) SAMD_EW_CASE(7) SAMD_EW_CASE(8)
+#undef SAMD_EW_CASE
+    default:
+      return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+template <typename W>
+cudaError_t swar_dispatch(samd_op op, int bits, const void *a, const void *b, void *out, int64_t nwords,
+                          int is_signed, int sat, int shift, cudaStream_t s) {
+  switch (op) {
+    case SAMD_ADD: return swar_dispatch_bits<W, SAMD_ADD>(bits, a, b, out, nwords, is_signed, sat, shift, s);
+    case SAMD_SUB: return swar_dispatch_bits<W, SAMD_SUB>(bits, a, b, out, nwords, is_signed, sat, shift, s);
+    case SAMD_MUL: return swar_dispatch_bits<W, SAMD_MUL>(bits, a, b, out, nwords, is_signed, sat, shift, s);
+    case SAMD_RELU: return swar_dispatch_bits<W, SAMD_RELU>(bits, a, b, out, nwords, is_signed, sat, shift, s);
+    default: return swar_dispatch_bits<W, SAMD_REQUANT>(bits, a, b, out, nwords, is_signed, sat, shift, s);
+  }
+}
+
+LaneFmt lane_fmt(samd_fmt f) {
+  return LaneFmt{f.bits, f.is_signed, f.bits + f.spacer, lanes_per_word(f)};
+}
+
+template <typename WI, typename WO>
+cudaError_t lane_dispatch(samd_op op, samd_fmt fa, const void *a, const void *b, samd_fmt fo, void *out, int64_t n,
+                          int shift, int sat, cudaStream_t s) {
+  int64_t nwo = words_per_row(fo, n);
+  int grid = grid_for(nwo, kThreads, sm_count() * 16);
+  ew_lane_kernel<WI, WO><<<grid, kThreads, 0, s>>>(static_cast<int>(op), lane_fmt(fa), static_cast<const WI *>(a),
+                                                   static_cast<const WI *>(b), lane_fmt(fo), static_cast<WO *>(out),
+                                                   n, nwo, shift, sat);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_elementwise(samd_op op, samd_fmt fa, const void *a, const void *b, samd_fmt fo, void *out,
+                               int64_t n, int shift, int saturate, cudaStream_t s) {
+  bool swar = same_fmt(fa, fo) && fa.spacer == 0;
+  if (swar) {
+    int64_t nwords = words_per_row(fa, n);
+    if (fa.word_bits == 32)
+      return swar_dispatch<uint32_t>(op, fa.bits, a, b, out, nwords, fa.is_signed, saturate, shift, s);
+    return swar_dispatch<uint64_t>(op, fa.bits, a, b, out, nwords, fa.is_signed, saturate, shift, s);
+  }
+  if (fa.word_bits == 32 && fo.word_bits == 32)
+    return lane_dispatch<uint32_t, uint32_t>(op, fa, a, b, fo, out, n, shift, saturate, s);
+  if (fa.word_bits == 32)
+    return lane_dispatch<uint32_t, uint64_t>(op, fa, a, b, fo, out, n, shift, saturate, s);
+  if (fo.word_bits == 32)
+    return lane_dispatch<uint64_t, uint32_t>(op, fa, a, b, fo, out, n, shift, saturate, s);
+  return lane_dispatch<uint64_t, uint64_t>(op, fa, a, b, fo, out, n, shift, saturate, s);
+}
+
+}  // namespace samd

@@ -1,0 +1,89 @@
+// samd_internal.cuh -- helpers shared by the libsamd translation units.
+//
+// Packed format (section 2.1 of the paper; Fig. 2 for spacer bits): lane i
+// of a row sits in word i / L at bit offset (i % L) * (bits + spacer), least
+// significant lane first; two's complement for signed lanes (section 6).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/samd.h"
+
+namespace samd {
+
+// ---- host-side format arithmetic -----------------------------------------
+
+inline bool fmt_valid(samd_fmt f) {
+  return f.bits >= 1 && f.bits <= 8 && f.spacer <= 8 && (f.word_bits == 32 || f.word_bits == 64) &&
+         f.is_signed <= 1 && f.bits + f.spacer <= f.word_bits;
+}
+
+inline int lanes_per_word(samd_fmt f) { return fmt_valid(f) ? f.word_bits / (f.bits + f.spacer) : 0; }
+
+inline int64_t words_per_row(samd_fmt f, int64_t inner) {
+  int L = lanes_per_word(f);
+  return (inner + L - 1) / L;
+}
+
+inline bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+inline bool same_fmt(samd_fmt a, samd_fmt b) {
+  return a.bits == b.bits && a.is_signed == b.is_signed && a.spacer == b.spacer && a.word_bits == b.word_bits;
+}
+
+inline int grid_for(int64_t work_items, int threads, int max_blocks) {
+  int64_t blocks = (work_items + threads - 1) / threads;
+  if (blocks < 1) blocks = 1;
+  if (blocks > max_blocks) blocks = max_blocks;
+  return static_cast<int>(blocks);
+}
+
+// Number of SMs of the current device (cached per device).
+int sm_count();
+
+// ---- device-side lane helpers ----------------------------------------------
+
+template <typename W>
+struct WordTraits;
+template <>
+struct WordTraits<uint32_t> {
+  static constexpr int kBits = 32;
+};
+template <>
+struct WordTraits<uint64_t> {
+  static constexpr int kBits = 64;
+};
+
+// Lane range of a b-bit lane.
+__host__ __device__ inline int lane_lo(int bits, bool is_signed) { return is_signed ? -(1 << (bits - 1)) : 0; }
+__host__ __device__ inline int lane_hi(int bits, bool is_signed) {
+  return is_signed ? (1 << (bits - 1)) - 1 : (1 << bits) - 1;
+}
+
+// Value of a lane pattern (low `bits` bits of p).
+__device__ __forceinline__ int lane_value(uint32_t p, int bits, bool is_signed) {
+  return is_signed ? (static_cast<int>(p << (32 - bits)) >> (32 - bits)) : static_cast<int>(p);
+}
+
+__device__ __forceinline__ int clamp_int(int v, int lo, int hi) { return v < lo ? lo : (v > hi ? hi : v); }
+
+}  // namespace samd
+
+// ---- launchers implemented in the kernel translation units ----------------
+
+namespace samd {
+cudaError_t launch_pack(samd_fmt f, const int8_t *src, void *dst, int64_t rows, int64_t inner, cudaStream_t s);
+cudaError_t launch_unpack(samd_fmt f, const void *src, int8_t *dst, int64_t rows, int64_t inner, cudaStream_t s);
+cudaError_t launch_elementwise(samd_op op, samd_fmt fa, const void *a, const void *b, samd_fmt fo, void *out,
+                               int64_t n, int shift, int saturate, cudaStream_t s);
+cudaError_t launch_maxpool2x2_nhwc(samd_fmt f, const void *in, void *out, int N, int C, int H, int W,
+                                   cudaStream_t s);
+
+struct ConvPlan;  // defined in conv2d.cuh
+samd_status conv2d_nhwc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
+                        int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, void *workspace,
+                        size_t workspace_bytes, cudaStream_t s);
+size_t conv2d_workspace_size(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw);
+cudaError_t read_device_status(int *status, int reset, cudaStream_t s);
+}  // namespace samd

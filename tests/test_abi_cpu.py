@@ -1,0 +1,89 @@
+"""The C-ABI library loads and exports every entry point include/samd.h
+declares; host-only queries and argument checks answer without a GPU (no
+compute call is made here)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_1809_10572_gb300 import build, samd
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "samd.h")
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"SAMD_API[^;(]*?\b(samd_\w+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    return samd.load()
+
+
+def test_header_declares_the_boundary():
+    names = declared_symbols()
+    for required in ("samd_pack", "samd_unpack", "samd_elementwise", "samd_conv2d", "samd_maxpool2x2"):
+        assert required in names
+    assert sorted(samd.EXPORTED) == names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_symbols():
+        assert hasattr(lib, name), name
+        assert ctypes.cast(getattr(lib, name), ctypes.c_void_p).value
+
+
+def test_library_is_built_in_tree_for_sm103a():
+    assert os.path.dirname(build.LIB).startswith(os.path.dirname(os.path.abspath(build.__file__)))
+    assert "arch=compute_103a,code=sm_103a" in build.ARCH
+
+
+def test_format_queries(lib):
+    for bits in range(1, 9):
+        for wb in (32, 64):
+            assert samd.samd_lanes_per_word(samd.fmt(bits, True, 0, wb)) == wb // bits
+            assert samd.samd_lanes_per_word(samd.fmt(bits, False, 1, wb)) == wb // (bits + 1)
+    f = samd.fmt(3, False)
+    assert samd.samd_packed_words(f, 7, 64) == 7 * 7
+    assert samd.samd_packed_words(f, 0, 64) == 0
+    assert samd.samd_packed_words(samd.fmt(9, False), 1, 1) == -1
+    assert samd.samd_packed_words(samd.fmt(4, False, 0, 16), 1, 1) == -1
+    assert samd.samd_lanes_per_word(samd.fmt(0, False)) == 0
+
+
+def test_invalid_arguments_are_rejected_before_any_launch(lib):
+    bad = samd.fmt(9, False)
+    assert lib.samd_pack(bad, None, None, 1, 1, None) == samd.SAMD_EINVAL
+    assert lib.samd_unpack(samd.fmt(4, False), None, None, -1, 4, None) == samd.SAMD_ESHAPE
+    assert lib.samd_pack(samd.fmt(4, False), None, None, 0, 5, None) == samd.SAMD_OK  # empty: nothing to do
+    assert lib.samd_pack(samd.fmt(4, False), None, None, 1, 5, None) == samd.SAMD_EINVAL
+    assert lib.samd_pack(samd.fmt(4, False), 16, 17, 1, 5, None) == samd.SAMD_EALIGN
+    f4 = samd.fmt(4, True)
+    assert lib.samd_elementwise(7, f4, None, None, f4, None, 1, 0, 0, None) == samd.SAMD_EINVAL
+    assert lib.samd_elementwise(samd.SAMD_ADD, f4, None, None, samd.fmt(3, True), None, 1, 0, 0, None) == samd.SAMD_EINVAL
+    assert lib.samd_elementwise(samd.SAMD_REQUANT, f4, None, None, f4, None, 1, 32, 0, None) == samd.SAMD_EINVAL
+    assert lib.samd_elementwise(samd.SAMD_ADD, f4, 16, None, f4, 16, 8, 0, 0, None) == samd.SAMD_EINVAL
+    assert lib.samd_elementwise(samd.SAMD_ADD, f4, 16, 32, f4, 8, 8, 0, 0, None) == samd.SAMD_EALIGN
+    assert lib.samd_maxpool2x2(f4, None, None, 1, 4, 3, 4, samd.SAMD_NHWC, None) == samd.SAMD_ESHAPE
+    assert lib.samd_maxpool2x2(f4, 16, 16, 1, 4, 4, 4, samd.SAMD_NCHW, None) == samd.SAMD_EUNSUP
+    assert lib.samd_status_str(samd.SAMD_EUNSUP).startswith(b"SAMD_EUNSUP")
+
+
+def test_conv_argument_checks(lib):
+    fa, fw = samd.fmt(4, False), samd.fmt(4, True)
+    d = samd.ConvShape(1, 16, 8, 8, 16).desc()
+    assert lib.samd_conv2d(None, fa, 16, fw, 16, 16, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_EINVAL
+    assert lib.samd_conv2d(ctypes.byref(d), fa, 16, fw, 16, None, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_EINVAL
+    nchw = samd.ConvShape(1, 16, 8, 8, 16).desc(samd.SAMD_NCHW)
+    assert lib.samd_conv2d(ctypes.byref(nchw), fa, 16, fw, 16, 16, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_EUNSUP
+    bad = samd.ConvShape(1, 16, 2, 2, 16, R=5, S=5, pad=1).desc()
+    assert lib.samd_conv2d(ctypes.byref(bad), fa, 16, fw, 16, 16, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_ESHAPE
+    # u8 x u8 over 3x3x64 taps breaks the 2^24 exactness bound of fp32 accumulation
+    big = samd.ConvShape(1, 64, 8, 8, 16).desc()
+    u8 = samd.fmt(8, False)
+    assert lib.samd_conv2d(ctypes.byref(big), u8, 16, u8, 16, 16, u8, None, 0, 16, 1 << 20, None) == samd.SAMD_EUNSUP
+    assert lib.samd_conv2d(ctypes.byref(d), fa, 16, fw, 24, 16, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_EALIGN
+    assert samd.samd_conv2d_workspace_size(d, fa, fw) > 0
+    assert samd.samd_conv2d_workspace_size(samd.ConvShape(1, 0, 8, 8, 16).desc(), fa, fw) == 0
