@@ -1,0 +1,509 @@
+#!/usr/bin/env python
+"""Benchmark of the bit-precise convolution hot path on GB300.
+
+Headline (one JSON line on rank 0): effective int MAC/s of the 3x3
+convolution N8 C64 -> 64 on 56x56 (pad 1) over the bit-width sweep -- lane
+widths b = 1..8 for activations and weights, all four signed/unsigned
+combinations, int32 accumulation requantized to a packed b-bit output. One
+step runs the 32 layers (one CUDA graph of 32 kernel launches). Weights are
+prepared once, as an inference deployment does at load time.
+
+Also reported: the packed elementwise ops (add, sub, mul, ReLU, requantize)
+plus pack/unpack and max-pool in GB/s on 2^28-lane arrays at every width;
+the conv kernel's roofline fraction; the same metric end to end through the
+C ABI from pinned host buffers; the CPU oracle timed on the host cores.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl samd|reference]
+                  [--workload sweep|vgg16|resnet50|conv1x]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+L2_FLUSH_BYTES = 512 << 20  # > 129 MB L2
+METRIC = "effective int MAC/s for b-bit conv2d vs bit width (fraction of int8 TC peak); packed-op GB/s"
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="samd", choices=["samd", "reference"])
+    ap.add_argument("--workload", default="sweep", choices=["sweep", "vgg16", "resnet50", "conv1x"])
+    ap.add_argument("--no-packed-ops", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--layers", type=str, default="", help="comma-separated layer indices (profiling aid)")
+    return ap.parse_args()
+
+
+# ---- distributed plumbing ------------------------------------------------------------
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+class Dist:
+    def __init__(self, backend):
+        import torch.distributed as dist
+
+        self.ws, self.rank, self.local = dist_env()
+        self.dist = dist if self.ws > 1 else None
+        if self.dist:
+            dist.init_process_group(backend)
+
+    def barrier(self):
+        if self.dist:
+            self.dist.barrier()
+
+    def max(self, x: float) -> float:
+        if not self.dist:
+            return x
+        import torch
+
+        t = torch.tensor([x], dtype=torch.float64, device="cuda" if self.dist.get_backend() == "nccl" else "cpu")
+        self.dist.all_reduce(t, op=self.dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.dist:
+            self.dist.destroy_process_group()
+
+
+# ---- clocks ------------------------------------------------------------------------------
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        out, _ = self.proc.communicate(timeout=10)
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax = float(parts[2])
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": smax, "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# ---- CPU oracle baseline ---------------------------------------------------------------
+
+def cpu_oracle_rate(layers, seconds: float):
+    """The oracle's direct convolution on one image of each layer in turn,
+    all host cores, until `seconds` have passed. Returns (MAC/s, threads, sample)."""
+    import oracle
+    from paper_1809_10572_gb300 import synth
+
+    threads = os.cpu_count() or 1
+    done_macs, t0, k = 0, time.perf_counter(), 0
+    names = []
+    while time.perf_counter() - t0 < seconds or k == 0:
+        layer = layers[k % len(layers)]
+        s = layer.shape
+        a = synth.lanes(synth.seed_for("cpu", k), (1, s.C, s.H, s.W), layer.ba, layer.sa)
+        w = synth.lanes(synth.seed_for("cpuw", k), (s.K, s.C, s.R, s.S), layer.bw, layer.sw)
+        oracle.conv2d(a, w, stride=s.stride, pad=s.pad, nthreads=threads)
+        done_macs += s.macs // s.N
+        names.append(layer.name)
+        k += 1
+    el = time.perf_counter() - t0
+    sample = f"{k} single-image layer runs ({', '.join(sorted(set(names))[:4])}{'...' if len(set(names)) > 4 else ''}), " \
+             f"{done_macs / 1e9:.2f} GMAC in {el:.1f} s"
+    return done_macs / el, threads, sample
+
+
+# ---- the reference arm: the CPU oracle ------------------------------------------------
+
+def run_reference(args, layers):
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    import oracle
+    from paper_1809_10572_gb300 import synth
+
+    threads = os.cpu_count() or 1
+    # one step = one image of each layer of the workload (a bounded sample)
+    inputs = []
+    for i, layer in enumerate(layers):
+        s = layer.shape
+        inputs.append((synth.lanes(synth.seed_for("ref", i), (1, s.C, s.H, s.W), layer.ba, layer.sa),
+                       synth.lanes(synth.seed_for("refw", i), (s.K, s.C, s.R, s.S), layer.bw, layer.sw), s))
+    step_macs = sum(s.macs // s.N for _, _, s in inputs)
+
+    def step():
+        for a, w, s in inputs:
+            oracle.conv2d(a, w, stride=s.stride, pad=s.pad, nthreads=threads)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    el = time.perf_counter() - t0
+    value = step_macs * args.steps / el
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "MAC/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+        "config": workload_config(args, layers),
+        "cpu_baseline": {"value": value, "unit": "MAC/s", "cores": threads, "kind": "oracle",
+                         "sample": f"one image of each of the {len(layers)} layers per step "
+                                   f"({step_macs / 1e9:.2f} GMAC/step)"},
+        "e2e": {"value": value, "unit": "MAC/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(args, layers):
+    from paper_1809_10572_gb300 import workloads
+
+    desc = {
+        "sweep": "3x3 conv N8 C64->64 56x56 pad1 stride1; act=weight=out width b in 1..8, signs uu/us/su/ss "
+                 "(32 layers), int32 acc requantized to packed b-bit; 32-bit words",
+        "vgg16": "VGG-16 13 conv layers 224x224 batch16, u4 act x s4 wt -> u4 (pools excluded from timing)",
+        "resnet50": "ResNet-50 v1.5 stage convs (52) batch64, u6 act x s2 wt -> u6",
+        "conv1x": "3x3 conv N1 C16->16 32x32, u4 x s4, 64-bit words",
+    }[args.workload]
+    return {"workload": desc, "layers": len(layers), "macs_per_step": workloads.total_macs(layers),
+            "l2": "flushed before every step (512 MiB write); inputs otherwise resident in HBM",
+            "weights": "prepared once into the fp16 operand layout (samd_conv2d_prepare), not in the step",
+            "launch": "one CUDA graph per step", "parallelism": f"replicas x{args.gpus}"}
+
+
+# ---- the samd arm ------------------------------------------------------------------------
+
+def build_layers(layers, dev):
+    import torch
+
+    from paper_1809_10572_gb300 import samd, synth, workloads
+
+    built = []
+    for i, layer in enumerate(layers):
+        s = layer.shape
+        fa = samd.fmt(layer.ba, layer.sa, 0, layer.word_bits)
+        fw = samd.fmt(layer.bw, layer.sw, 0, layer.word_bits)
+        fo = samd.fmt(layer.bo, layer.so, 0, layer.word_bits)
+        a = synth.lanes_t(synth.seed_for("bench", i), (s.N * s.H * s.W, s.C), layer.ba, layer.sa, device=dev)
+        a_w = samd.pack(synth.to_bytes_t(a), fa)
+        del a
+        w = synth.lanes_t(synth.seed_for("benchw", i), (s.K * s.R * s.S, s.C), layer.bw, layer.sw, device=dev)
+        w_w = samd.pack(synth.to_bytes_t(w), fw)
+        conv = samd.PreparedConv(w_w, s, fa, fw, fo)
+        _, out = conv.outputs(want_acc=False)
+        shift = workloads.harness_shift(layer.ba, layer.bw, layer.bo, s.C * s.R * s.S)
+        built.append({"layer": layer, "conv": conv, "act": a_w, "out": out, "shift": shift})
+    torch.cuda.synchronize()
+    return built
+
+
+def time_packed_ops(dev, flush):
+    """GB/s of pack/unpack, the five elementwise ops and max-pool at 2^28 lanes."""
+    import torch
+
+    from paper_1809_10572_gb300 import samd, synth, workloads
+
+    n = workloads.ELEMENTWISE_N
+    res = {}
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    def timed(fn, nbytes, reps=3):
+        ts = []
+        for _ in range(reps):
+            flush()
+            start.record()
+            fn()
+            end.record()
+            end.synchronize()
+            ts.append(start.elapsed_time(end) * 1e-3)
+        return nbytes / statistics.median(ts) / 1e9
+
+    launches = 0
+    for signed in (False, True):
+        tag = "s" if signed else "u"
+        for b in range(1, 9):
+            f = samd.fmt(b, signed)
+            xb = synth.to_bytes_t(synth.lanes_t(synth.seed_for("ewx", b, signed), (n,), b, signed, device=dev))
+            xw = samd.pack(xb, f)
+            yw = samd.pack(synth.to_bytes_t(synth.lanes_t(synth.seed_for("ewy", b, signed), (n,), b, signed,
+                                                          device=dev)), f)
+            out = torch.empty_like(xw)
+            wbytes = xw.numel() * 4
+            res.setdefault("pack", {}).setdefault(tag, []).append(
+                timed(lambda: samd.samd_pack(f, xb, out, 1, n), n + wbytes))
+            res.setdefault("unpack", {}).setdefault(tag, []).append(
+                timed(lambda: samd.samd_unpack(f, xw, xb, 1, n), n + wbytes))
+            for op in workloads.ELEMENTWISE_OPS:
+                binary = op in ("add", "sub", "mul")
+                nb = (3 if binary else 2) * wbytes
+                res.setdefault(op, {}).setdefault(tag, []).append(
+                    timed(lambda: samd.samd_elementwise(op, f, xw, yw if binary else None, f, out, n,
+                                                        1 if op == "requant" else 0, 0), nb))
+            launches += 3 * 7
+            del xb, xw, yw, out
+    # 2x2 max-pool on the largest VGG-16 activation (16 x 224 x 224 x 64, u4)
+    f = samd.fmt(4, False)
+    N, C, H, W = 16, 64, 224, 224
+    xw = samd.pack(synth.to_bytes_t(synth.lanes_t(5, (N * H * W, C), 4, False, device=dev)), f)
+    out = samd.empty_words(f, N * H * W // 4, C, dev)
+    nb = (xw.numel() + out.numel()) * 4
+    res["maxpool2x2"] = {"u": [timed(lambda: samd.samd_maxpool2x2(f, xw, out, N, C, H, W), nb)]}
+    return res
+
+
+def run_samd(args, layers):
+    import torch
+
+    import oracle  # noqa: F401  (CPU-baseline leg only)
+    from paper_1809_10572_gb300 import samd, workloads
+
+    ws, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    d = Dist("nccl")
+    samd.load()
+
+    built = build_layers(layers, dev)
+    step_macs = workloads.total_macs(layers)
+    flush_buf = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    def flush():
+        flush_buf.fill_(1)
+
+    stream = torch.cuda.Stream(device=dev)
+
+    def step_calls(s):
+        for b in built:
+            b["conv"](b["act"], None, b["out"], b["shift"], stream=s)
+
+    # first calls outside any capture (kernel attributes, tensor-map entry point)
+    with torch.cuda.stream(stream):
+        step_calls(stream)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        step_calls(torch.cuda.current_stream())
+    torch.cuda.synchronize()
+    if samd.samd_device_status() != 0:
+        raise RuntimeError("a kernel recorded a timeout")
+
+    # warm-up
+    for _ in range(args.warmup):
+        flush()
+        graph.replay()
+    torch.cuda.synchronize()
+
+    # timed region: K steps, L2 flushed between steps (outside the events)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    if rank == 0:
+        clocks.start()
+    d.barrier()
+    torch.cuda.synchronize()
+    t_wall = time.perf_counter()
+    cur = torch.cuda.current_stream()
+    for i in range(args.steps):
+        flush()
+        ev[i][0].record(cur)
+        graph.replay()
+        ev[i][1].record(cur)
+    torch.cuda.synchronize()
+    d.barrier()
+    wall = time.perf_counter() - t_wall
+    clk = clocks.stop() if rank == 0 else None
+    step_s = [a.elapsed_time(b) * 1e-3 for a, b in ev]
+    dev_time = d.max(sum(step_s))
+    if samd.samd_device_status() != 0:
+        raise RuntimeError("a kernel recorded a timeout")
+    value = step_macs * args.steps * ws / dev_time
+    ms_per_step = dev_time / args.steps * 1e3
+
+    # per-layer throughput (one graph per layer, replayed with events)
+    by_layer = {}
+    for b in built:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            b["conv"](b["act"], None, b["out"], b["shift"], stream=torch.cuda.current_stream())
+        ts = []
+        for _ in range(5):
+            flush()
+            s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            s0.record(cur)
+            g.replay()
+            s1.record(cur)
+            s1.synchronize()
+            ts.append(s0.elapsed_time(s1) * 1e-3)
+        by_layer[b["layer"].name] = b["layer"].macs / statistics.median(ts)
+
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except (OSError, ValueError):
+        pass
+    bf16_peak = peaks.get("bf16_tflops")
+    peak_src = "measured (bf16 burst; the fp16 dense rate equals bf16)" if bf16_peak else "fallback"
+    bf16_peak = bf16_peak or 1900.0
+    achieved_tflops = 2.0 * step_macs / (ms_per_step * 1e-3) / 1e12
+    roofline = {"kernel": "conv_tc_kernel", "bound": "tensor", "achieved": achieved_tflops, "peak": bf16_peak,
+                "unit": "TFLOP/s", "frac": achieved_tflops / bf16_peak, "traffic": None,
+                "peak_source": peak_src,
+                "note": "achieved = 2 x direct-conv MACs per launch / mean launch time (graph step time / launches)"}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "MAC/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f16 x f16 -> f32 tensor-core MMA on exact integers (b-bit packed lanes)", "data": "synthetic",
+        "config": workload_config(args, layers), "wall_s_timed_region": wall,
+        "gpu_launches": args.steps * len(built),
+        "roofline": roofline,
+    }
+    if args.workload == "sweep":
+        per_bits = {}
+        for name, v in by_layer.items():
+            per_bits.setdefault(name.split("_")[0], []).append(v)
+        line["by_bits_mac_s"] = {k: statistics.mean(v) for k, v in per_bits.items()}
+    line["by_layer_mac_s"] = by_layer
+
+    # int8 tensor-core peak (for the metric's "fraction of int8 TC peak")
+    if rank == 0:
+        line["int8_tc_peak"] = measure_int8_peak(dev)
+        if line["int8_tc_peak"].get("tops"):
+            line["frac_of_int8_tc_peak"] = 2 * value / ws / (line["int8_tc_peak"]["tops"] * 1e12)
+
+    # e2e: the same step through the C ABI from pinned host buffers
+    if not args.no_e2e:
+        line["e2e"] = measure_e2e(built, step_macs, args, dev, ws, d)
+
+    if rank == 0 and not args.no_packed_ops:
+        ops = time_packed_ops(dev, flush)
+        hbm = peaks.get("hbm_gbs") or 6800.0
+        fr = [v / hbm for op, sg in ops.items() for vals in sg.values() for v in vals]
+        line["packed_ops_gb_s"] = ops
+        line["packed_ops_roofline"] = {"bound": "hbm", "peak": hbm, "unit": "GB/s",
+                                       "peak_source": "measured" if peaks.get("hbm_gbs") else "fallback",
+                                       "min_frac": min(fr), "median_frac": statistics.median(fr), "max_frac": max(fr),
+                                       "n": 2 ** 28, "word_bits": 32,
+                                       "bytes": "each input word read once + each output word written once"}
+    line["clocks"] = clk
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        v, cores, sample = cpu_oracle_rate(layers, args.cpu_seconds)
+        line["cpu_baseline"] = {"value": v, "unit": "MAC/s", "cores": cores, "kind": "oracle", "sample": sample}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    d.close()
+    return 0
+
+
+def measure_int8_peak(dev):
+    import torch
+
+    try:
+        n = 8192
+        a = torch.randint(-128, 127, (n, n), dtype=torch.int8, device=dev)
+        b = torch.randint(-128, 127, (n, n), dtype=torch.int8, device=dev)
+        torch._int_mm(a, b)
+        torch.cuda.synchronize()
+        best = None
+        for _ in range(5):
+            s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            s0.record()
+            torch._int_mm(a, b)
+            s1.record()
+            s1.synchronize()
+            t = s0.elapsed_time(s1) * 1e-3
+            best = t if best is None else min(best, t)
+        return {"tops": 2 * n ** 3 / best / 1e12, "how": "torch._int_mm int8 8192^3, best of 5"}
+    except Exception as e:  # noqa: BLE001
+        return {"tops": None, "how": f"torch._int_mm unavailable: {type(e).__name__}"}
+
+
+def measure_e2e(built, step_macs, args, dev, ws, d):
+    import torch
+
+    host_in = [torch.empty(b["act"].shape, dtype=b["act"].dtype, pin_memory=True) for b in built]
+    host_out = [torch.empty(b["out"].shape, dtype=b["out"].dtype, pin_memory=True) for b in built]
+    for h, b in zip(host_in, built):
+        h.copy_(b["act"])
+    dev_in = [torch.empty_like(b["act"]) for b in built]
+    h2d = sum(t.numel() * t.element_size() for t in host_in)
+    d2h = sum(t.numel() * t.element_size() for t in host_out)
+    s = torch.cuda.current_stream()
+
+    def step():
+        for b, hi, di, ho in zip(built, host_in, dev_in, host_out):
+            di.copy_(hi, non_blocking=True)
+            b["conv"](di, None, b["out"], b["shift"], stream=s)
+            ho.copy_(b["out"], non_blocking=True)
+        s.synchronize()
+
+    for _ in range(max(1, args.warmup)):
+        step()
+    d.barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    el = d.max(time.perf_counter() - t0)
+    return {"value": step_macs * args.steps * ws / el, "unit": "MAC/s", "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "how": "per layer: pinned H2D of packed act, samd_conv2d_prepared, "
+                                               "pinned D2H of packed output; sync per step"}
+
+
+def main():
+    args = parse_args()
+    from paper_1809_10572_gb300 import workloads
+
+    layers = workloads.WORKLOADS[args.workload]()
+    if args.layers:
+        idx = [int(t) for t in args.layers.split(",")]
+        layers = [layers[i] for i in idx]
+    if args.impl == "reference":
+        return run_reference(args, layers)
+    return run_samd(args, layers)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

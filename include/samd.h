@@ -154,10 +154,12 @@ typedef struct {
  * workspace / workspace_bytes: caller-owned device scratch of at least
  * samd_conv2d_workspace_size(...) bytes (16-byte aligned) that receives the
  * weights in the tensor-core operand layout on every call.
- * Limits (SAMD_EUNSUP beyond them): spacer 0 for fa and fw; R, S <= 16;
- * and the exactness bound of the accumulation, R*S*C * max|a| * max|w| <
- * 2^24 (or < 2^24 * 16 with an unsigned 8-bit or signed 8-bit act, split in
- * two 4-bit digits).
+ * Exactness: the sum runs on the tensor cores over fp16 operands with fp32
+ * accumulation, exact while every partial sum stays below 2^24. If
+ * R*S*C * max|a| * max|w| reaches 2^24 and the weights have 5-8 bits, the
+ * weights are split into two 4-bit digits (two exact accumulators per
+ * output); if R*S*C * max|a| * 16 also reaches 2^24, SAMD_EUNSUP.
+ * Other limits (SAMD_EUNSUP): spacer 0 for fa and fw; R, S <= 16.
  * A kernel that gives up on a bounded wait leaves its outputs undefined and
  * records SAMD_ETIMEOUT for samd_device_status.
  */
@@ -165,8 +167,27 @@ SAMD_API samd_status samd_conv2d(const samd_conv_desc *desc, samd_fmt fa, const 
                         int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, void *workspace,
                         size_t workspace_bytes, samd_stream_t stream);
 
-/* Bytes of workspace samd_conv2d needs for this shape and formats (0 on error). */
+/* Bytes of workspace samd_conv2d needs for this shape and formats, for any
+ * output format (0 on error). The same size suffices for
+ * samd_conv2d_prepare. */
 SAMD_API size_t samd_conv2d_workspace_size(const samd_conv_desc *desc, samd_fmt fa, samd_fmt fw);
+
+/*
+ * Weights prepared once, used by many calls (the weights of an inference
+ * layer do not change between batches). samd_conv2d_prepare widens the
+ * packed weights wt ([K][R][S][C] along C, format fw) into `prepared`
+ * (caller-owned, >= samd_conv2d_workspace_size bytes, 16-byte aligned);
+ * samd_conv2d_prepared then runs the convolution of samd_conv2d without
+ * touching wt, in one kernel launch. Both calls must get the same desc, fa,
+ * fw and fo; fo may be {0,0,0,0} ("no packed output") in both. The
+ * prepared buffer is only read by samd_conv2d_prepared, so concurrent calls
+ * may share it.
+ */
+SAMD_API samd_status samd_conv2d_prepare(const samd_conv_desc *desc, samd_fmt fa, samd_fmt fw, const void *wt,
+                                         samd_fmt fo, void *prepared, size_t prepared_bytes, samd_stream_t stream);
+SAMD_API samd_status samd_conv2d_prepared(const samd_conv_desc *desc, samd_fmt fa, const void *act, samd_fmt fw,
+                                          const void *prepared, size_t prepared_bytes, int32_t *acc_out,
+                                          samd_fmt fo, void *packed_out, int shift, samd_stream_t stream);
 
 /*
  * samd_maxpool2x2: lane-wise max over 2x2 windows with stride 2 (used

@@ -15,8 +15,10 @@
 // Exactness. tcgen05 has no integer MMA on sm_103a, so lanes are widened to
 // fp16, which holds every integer of [-128, 255] exactly; products are exact
 // and the fp32 accumulators hold exact integers while every partial sum
-// stays below 2^24. The host only launches shapes whose bound
-// R*S*C*max|a|*max|w| is below 2^24.
+// stays below 2^24. When R*S*C*max|a|*max|w| reaches 2^24 (wide weights over
+// many taps), the weights are split into two 4-bit digits w = 16*hi + lo,
+// stacked along the MMA's N: one MMA fills two accumulator halves, each far
+// below 2^24, and the epilogue forms 16*hi + lo in int32.
 //
 // CTA = 6 warps, one 128-pixel tile x one block of output channels:
 //   warp 0      TMEM allocation; lane 0 streams weight tiles with TMA
@@ -25,8 +27,9 @@
 //               widen them to fp16 in the 128-byte-swizzled K-major layout,
 //               then run the epilogue: tcgen05.ld of the fp32 accumulators,
 //               int32 store and/or requantize-and-pack to fo.
-// Weights are widened once per call into the workspace (a [K][Kg] fp16
-// matrix in the same Kg order) by wprep_kernel.
+// Weights are widened into a [K][Kg] fp16 matrix in the same Kg order by
+// wprep_kernel: once per call (samd_conv2d), or once for many calls
+// (samd_conv2d_prepare + samd_conv2d_prepared).
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
@@ -75,7 +78,9 @@ struct ConvArgs {
   int words_total;  // R * S * wpr: reduction length in packed words
   int nchunks;      // ceil(words_total / words per chunk)
   int NBc;          // output channels per channel block
-  int n_mma;        // MMA N (NBc rounded up to 16)
+  int n_mma;        // NBc rounded up to 16
+  int mma_n;        // MMA N: n_mma, or 2 * n_mma with split weight digits
+  int split;        // 1: accumulator columns [0, n_mma) hold hi digits, [n_mma, 2 n_mma) lo digits
   int stages;
   uint32_t tmem_cols;
   int out_bits, out_signed, out_lane_w, out_L, out_word64, out_wpr;
@@ -200,7 +205,7 @@ __global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_const
   __shared__ int s_skip;
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int ST = args.stages;
-  const uint32_t b_bytes = static_cast<uint32_t>(args.n_mma) * 128u;
+  const uint32_t b_bytes = static_cast<uint32_t>(args.mma_n) * 128u;
   uint8_t *sA = smem;
   uint8_t *sB = smem + ST * kATileBytes;
   uint64_t *bars = reinterpret_cast<uint64_t *>(sB + ST * b_bytes);
@@ -252,7 +257,7 @@ __global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_const
           break;
         }
         ptx::mbar_arrive_expect_tx(full_b(s), b_bytes);
-        ptx::tma_load_2d(ptx::smem_addr(sB + s * b_bytes), &tmap_b, c * BK, nb * args.n_mma, full_b(s));
+        ptx::tma_load_2d(ptx::smem_addr(sB + s * b_bytes), &tmap_b, c * BK, nb * args.mma_n, full_b(s));
         issued = c + 1;
       }
       if (!ok) {
@@ -265,7 +270,7 @@ __global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_const
   } else if (warp == 1) {
     if (lane == 0) {
       // ---- MMA issue ----
-      const uint32_t idesc = ptx::idesc_f16_f32(BM, args.n_mma);
+      const uint32_t idesc = ptx::idesc_f16_f32(BM, args.mma_n);
       for (int c = 0; c < args.nchunks; ++c) {
         const int s = c % ST, round = c / ST;
         if (!ptx::mbar_wait_bounded(full_a(s), round & 1, status, kWaitLimitNs) ||
@@ -343,13 +348,19 @@ __global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_const
       long long widx = g.row_valid && args.packed_out ? m * args.out_wpr + ch0 / args.out_L : 0;
       for (int col = 0; col < nvalid; col += 32) {
         uint32_t r[32];
+        int v[32];
         ptx::tmem_ld_32x32b_x32(taddr + col, r);
         ptx::tmem_wait_ld();
-        if (!g.row_valid) continue;
-        const int cnt = nvalid - col < 32 ? nvalid - col : 32;
-        int v[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) v[i] = __float2int_rn(__uint_as_float(r[i]));
+        if (args.split) {  // acc = 16 * hi + lo
+          ptx::tmem_ld_32x32b_x32(taddr + args.n_mma + col, r);
+          ptx::tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = 16 * v[i] + __float2int_rn(__uint_as_float(r[i]));
+        }
+        if (!g.row_valid) continue;
+        const int cnt = nvalid - col < 32 ? nvalid - col : 32;
         if (args.acc_out) {
           int32_t *dst = args.acc_out + m * args.K + ch0 + col;
           if (cnt == 32 && vec_ok) {
@@ -403,7 +414,7 @@ struct WPrepArgs {
   int K, C, RS;
   int bits_w, signed_w, lane_w_w, Lw, wpr_w;  // weight format
   int bits_a, La, WC, wpr_a, words_total;      // reduction order set by the activation format
-  int Kpad, n_mma, NBc;
+  int Kpad, n_mma, mma_n, NBc, split;
   long long rows_total;
 };
 
@@ -416,7 +427,9 @@ __global__ void __launch_bounds__(256) wprep_kernel(const WW *__restrict__ wt, _
        idx += (long long)gridDim.x * blockDim.x) {
     const long long rowi = idx / a.Kpad;
     const int kpos = static_cast<int>(idx - rowi * a.Kpad);
-    const int nb = static_cast<int>(rowi / a.n_mma), r = static_cast<int>(rowi % a.n_mma);
+    const int nb = static_cast<int>(rowi / a.mma_n), rb = static_cast<int>(rowi % a.mma_n);
+    const int plane = a.split ? rb / a.n_mma : -1;  // 0: high digit, 1: low digit
+    const int r = a.split ? rb % a.n_mma : rb;
     const int k = nb * a.NBc + r;
     const int chunk = kpos / BK, j = kpos % BK;
     const int q = j / a.La, pos = j % a.La;
@@ -431,6 +444,8 @@ __global__ void __launch_bounds__(256) wprep_kernel(const WW *__restrict__ wt, _
           const WW word = wt[wrow * a.wpr_w + ch / a.Lw];
           const uint32_t p = static_cast<uint32_t>(word >> ((ch % a.Lw) * a.lane_w_w)) & mask;
           v = lane_value(p, a.bits_w, a.signed_w);
+          if (plane == 0) v >>= 4;       // floor(v / 16)
+          else if (plane == 1) v &= 15;  // v - 16 * floor(v / 16)
         }
       }
     }
@@ -459,18 +474,29 @@ EncodeTiledFn encode_tiled() {
 }
 
 struct Plan {
-  int wpr, words_total, La, WC, nchunks, Kpad, NBc, n_mma, nblocks, stages, Ho, Wo;
+  int wpr, words_total, La, WC, nchunks, Kpad, NBc, n_mma, mma_n, split, nblocks, stages, Ho, Wo;
   long long M;
   uint32_t tmem_cols;
   size_t smem_bytes;
   size_t ws_bytes;
 };
 
-int lanes_of(samd_fmt f) { return lanes_per_word(f); }
+long long max_abs(samd_fmt f) { return f.is_signed ? (1LL << (f.bits - 1)) : ((1LL << f.bits) - 1); }
 
-bool make_plan(const samd_conv_desc *d, samd_fmt fa, const samd_fmt *fo_or_null, Plan &p) {
-  p.La = lanes_of(fa);
-  if (p.La == 0) return false;
+// Tiling, reduction order and exactness mode for one convolution. fo.bits == 0
+// means no packed output. Returns SAMD_EUNSUP when no mode keeps every
+// accumulator below 2^24.
+samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fmt fo, Plan &p) {
+  p.La = lanes_per_word(fa);
+  if (p.La == 0) return SAMD_EINVAL;
+  const long long taps = static_cast<long long>(d->R) * d->S * d->C;
+  const long long bound = taps * max_abs(fa) * max_abs(fw);
+  p.split = 0;
+  if (bound >= (1LL << 24)) {
+    // two 4-bit weight digits: each accumulator sums at most taps * max|a| * 16
+    if (fw.bits <= 4 || taps * max_abs(fa) * 16 >= (1LL << 24)) return SAMD_EUNSUP;
+    p.split = 1;
+  }
   p.WC = BK / p.La;
   p.wpr = static_cast<int>((d->C + p.La - 1) / p.La);
   p.words_total = d->R * d->S * p.wpr;
@@ -479,33 +505,66 @@ bool make_plan(const samd_conv_desc *d, samd_fmt fa, const samd_fmt *fo_or_null,
   p.Ho = (d->H + 2 * d->pad - d->R) / d->stride + 1;
   p.Wo = (d->W + 2 * d->pad - d->S) / d->stride + 1;
   p.M = static_cast<long long>(d->N) * p.Ho * p.Wo;
-  if (d->K <= 256) {
+  // A channel block must cover whole output words so that no packed word is
+  // shared by two CTAs.
+  const int limit = p.split ? 128 : 256;
+  if (d->K <= limit) {
     p.NBc = d->K;
   } else {
-    int Lo = fo_or_null ? lanes_of(*fo_or_null) : 1;
-    p.NBc = (256 / Lo) * Lo;
+    const int Lo = fo.bits ? lanes_per_word(fo) : 1;
+    p.NBc = (limit / Lo) * Lo;
   }
   p.n_mma = (p.NBc + 15) / 16 * 16;
+  p.mma_n = p.split ? 2 * p.n_mma : p.n_mma;
   p.nblocks = (d->K + p.NBc - 1) / p.NBc;
   uint32_t cols = 32;
-  while (cols < static_cast<uint32_t>(p.n_mma)) cols <<= 1;
+  while (cols < static_cast<uint32_t>(p.mma_n)) cols <<= 1;
   p.tmem_cols = cols;
-  const size_t stage_bytes = kATileBytes + static_cast<size_t>(p.n_mma) * 128;
+  const size_t stage_bytes = kATileBytes + static_cast<size_t>(p.mma_n) * 128;
   int st = static_cast<int>((100 * 1024) / stage_bytes);
   if (st < 2) st = 2;
   if (st > 6) st = 6;
   p.stages = st;
   p.smem_bytes = 1024 + st * stage_bytes + (3 * st + 2) * 8 + 16;
-  p.ws_bytes = static_cast<size_t>(p.nblocks) * p.n_mma * p.Kpad * sizeof(__half);
-  return true;
+  p.ws_bytes = static_cast<size_t>(p.nblocks) * p.mma_n * p.Kpad * sizeof(__half);
+  return SAMD_OK;
+}
+
+// cudaFuncSetAttribute once per (kernel, device), so that launches made
+// while a stream is being captured into a graph issue no other CUDA call.
+cudaError_t ensure_smem_attr(const void *kern, size_t smem) {
+  static std::mutex mu;
+  static const void *done_fn[256];
+  static int done_dev[256];
+  static size_t done_smem[256];
+  static int n_done = 0;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  for (int i = 0; i < n_done; ++i)
+    if (done_fn[i] == kern && done_dev[i] == dev && done_smem[i] >= smem) return cudaSuccess;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+  if (e != cudaSuccess) return e;
+  for (int i = 0; i < n_done; ++i)
+    if (done_fn[i] == kern && done_dev[i] == dev) {
+      done_smem[i] = 200 * 1024;
+      return cudaSuccess;
+    }
+  if (n_done < 256) {
+    done_fn[n_done] = kern;
+    done_dev[n_done] = dev;
+    done_smem[n_done] = 200 * 1024;
+    ++n_done;
+  }
+  return cudaSuccess;
 }
 
 template <typename W, int BITS, bool SIGNED>
 cudaError_t launch_conv_variant(const CUtensorMap &tmap, const ConvArgs &args, dim3 grid, size_t smem,
                                 cudaStream_t s) {
   auto kern = conv_tc_kernel<W, BITS, SIGNED>;
-  // the attribute is per function and device; setting it again is harmless
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  cudaError_t e = ensure_smem_attr(reinterpret_cast<const void *>(kern), smem);
   if (e != cudaSuccess) return e;
   kern<<<grid, kThreads, smem, s>>>(tmap, args);
   return cudaGetLastError();
@@ -528,36 +587,37 @@ cudaError_t launch_conv_word(samd_fmt fa, const CUtensorMap &tmap, const ConvArg
   }
 }
 
+samd_fmt none_fmt() { return samd_fmt{0, 0, 0, 0}; }
+
 }  // namespace
 
 size_t conv2d_workspace_size(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw) {
-  (void)fw;
+  // the channel blocking depends on the output format only above 128/256
+  // channels: report the largest size over every output format
   Plan p;
-  if (!make_plan(d, fa, nullptr, p)) return 0;
-  // the channel blocking depends on the output format only above 256
-  // channels; reserve the largest layout (one lane per word block)
-  if (d->K > 256) {
-    Plan q = p;
-    q.NBc = 250;  // smallest block any output format yields (10 lanes per word)
-    q.n_mma = 256;
-    q.nblocks = (d->K + q.NBc - 1) / q.NBc;
-    size_t big = static_cast<size_t>(q.nblocks) * q.n_mma * q.Kpad * sizeof(__half);
-    return big > p.ws_bytes ? big : p.ws_bytes;
-  }
-  return p.ws_bytes;
+  if (make_plan(d, fa, fw, none_fmt(), p) != SAMD_OK) return 0;
+  size_t best = p.ws_bytes;
+  for (int wb : {32, 64})
+    for (int bits = 1; bits <= 8; ++bits)
+      for (int sp = 0; sp + bits <= 16 && sp <= 8; ++sp) {
+        samd_fmt fo{static_cast<uint8_t>(bits), 0, static_cast<uint8_t>(sp), static_cast<uint8_t>(wb)};
+        Plan q;
+        if (make_plan(d, fa, fw, fo, q) == SAMD_OK && q.ws_bytes > best) best = q.ws_bytes;
+      }
+  return best;
 }
 
-samd_status conv2d_nhwc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
-                        int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, void *workspace,
-                        size_t workspace_bytes, cudaStream_t s) {
+samd_status conv2d_check(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw) {
   Plan p;
-  if (!make_plan(d, fa, packed_out ? &fo : nullptr, p)) return SAMD_EINVAL;
-  if (workspace_bytes < p.ws_bytes) return SAMD_ESHAPE;
-  if (p.M == 0) return SAMD_OK;
-  EncodeTiledFn enc = encode_tiled();
-  if (!enc) return SAMD_ECUDA;
+  return make_plan(d, fa, fw, none_fmt(), p);
+}
 
-  // 1. widen the weights into the reduction order of the activations
+samd_status conv2d_prepare(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const void *wt, samd_fmt fo,
+                           void *prepared, size_t prepared_bytes, cudaStream_t s) {
+  Plan p;
+  samd_status st = make_plan(d, fa, fw, fo, p);
+  if (st != SAMD_OK) return st;
+  if (prepared_bytes < p.ws_bytes) return SAMD_ESHAPE;
   WPrepArgs wa;
   wa.K = d->K;
   wa.C = d->C;
@@ -574,32 +634,44 @@ samd_status conv2d_nhwc(const samd_conv_desc *d, samd_fmt fa, const void *act, s
   wa.words_total = p.words_total;
   wa.Kpad = p.Kpad;
   wa.n_mma = p.n_mma;
+  wa.mma_n = p.mma_n;
   wa.NBc = p.NBc;
-  wa.rows_total = static_cast<long long>(p.nblocks) * p.n_mma;
-  __half *B = static_cast<__half *>(workspace);
-  {
-    const long long total = wa.rows_total * wa.Kpad;
-    const int grid = grid_for(total, 256, sm_count() * 8);
-    if (fw.word_bits == 32)
-      wprep_kernel<uint32_t><<<grid, 256, 0, s>>>(static_cast<const uint32_t *>(wt), B, wa);
-    else
-      wprep_kernel<uint64_t><<<grid, 256, 0, s>>>(static_cast<const uint64_t *>(wt), B, wa);
-    if (cudaGetLastError() != cudaSuccess) return SAMD_ECUDA;
-  }
+  wa.split = p.split;
+  wa.rows_total = static_cast<long long>(p.nblocks) * p.mma_n;
+  const long long total = wa.rows_total * wa.Kpad;
+  const int grid = grid_for(total, 256, sm_count() * 8);
+  __half *B = static_cast<__half *>(prepared);
+  if (fw.word_bits == 32)
+    wprep_kernel<uint32_t><<<grid, 256, 0, s>>>(static_cast<const uint32_t *>(wt), B, wa);
+  else
+    wprep_kernel<uint64_t><<<grid, 256, 0, s>>>(static_cast<const uint64_t *>(wt), B, wa);
+  return cudaGetLastError() == cudaSuccess ? SAMD_OK : SAMD_ECUDA;
+}
 
-  // 2. tensor map over the widened weights: [rows_total][Kpad] fp16, tiles of
-  //    n_mma rows x 64 elements, 128-byte swizzle
+samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const void *act, const void *prepared,
+                       size_t prepared_bytes, int32_t *acc_out, samd_fmt fo, void *packed_out, int shift,
+                       cudaStream_t s) {
+  Plan p;
+  samd_status st = make_plan(d, fa, fw, fo, p);
+  if (st != SAMD_OK) return st;
+  if (prepared_bytes < p.ws_bytes) return SAMD_ESHAPE;
+  if (p.M == 0) return SAMD_OK;
+  EncodeTiledFn enc = encode_tiled();
+  if (!enc) return SAMD_ECUDA;
+
+  // tensor map over the widened weights: [nblocks * mma_n][Kpad] fp16, tiles
+  // of mma_n rows x 64 elements, 128-byte swizzle
   CUtensorMap tmap;
-  cuuint64_t gdim[2] = {static_cast<cuuint64_t>(p.Kpad), static_cast<cuuint64_t>(wa.rows_total)};
+  const long long rows_total = static_cast<long long>(p.nblocks) * p.mma_n;
+  cuuint64_t gdim[2] = {static_cast<cuuint64_t>(p.Kpad), static_cast<cuuint64_t>(rows_total)};
   cuuint64_t gstride[1] = {static_cast<cuuint64_t>(p.Kpad) * sizeof(__half)};
-  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(p.n_mma)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(p.mma_n)};
   cuuint32_t estride[2] = {1, 1};
-  CUresult cr = enc(&tmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, workspace, gdim, gstride, box, estride,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult cr = enc(&tmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(prepared), gdim, gstride, box,
+                    estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (cr != CUDA_SUCCESS) return SAMD_ECUDA;
 
-  // 3. the convolution
   ConvArgs a;
   a.act = act;
   a.acc_out = acc_out;
@@ -621,6 +693,8 @@ samd_status conv2d_nhwc(const samd_conv_desc *d, samd_fmt fa, const void *act, s
   a.nchunks = p.nchunks;
   a.NBc = p.NBc;
   a.n_mma = p.n_mma;
+  a.mma_n = p.mma_n;
+  a.split = p.split;
   a.stages = p.stages;
   a.tmem_cols = p.tmem_cols;
   a.out_bits = packed_out ? fo.bits : 8;
@@ -634,6 +708,15 @@ samd_status conv2d_nhwc(const samd_conv_desc *d, samd_fmt fa, const void *act, s
   cudaError_t e = fa.word_bits == 32 ? launch_conv_word<uint32_t>(fa, tmap, a, grid, p.smem_bytes, s)
                                      : launch_conv_word<uint64_t>(fa, tmap, a, grid, p.smem_bytes, s);
   return e == cudaSuccess ? SAMD_OK : SAMD_ECUDA;
+}
+
+samd_status conv2d_nhwc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
+                        int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, void *workspace,
+                        size_t workspace_bytes, cudaStream_t s) {
+  const samd_fmt fplan = packed_out ? fo : none_fmt();
+  samd_status st = conv2d_prepare(d, fa, fw, wt, fplan, workspace, workspace_bytes, s);
+  if (st != SAMD_OK) return st;
+  return conv2d_run(d, fa, fw, act, workspace, workspace_bytes, acc_out, fplan, packed_out, shift, s);
 }
 
 cudaError_t read_device_status(int *status, int reset, cudaStream_t s) {

@@ -25,9 +25,6 @@ namespace {
 
 samd_status from_cuda(cudaError_t e) { return e == cudaSuccess ? SAMD_OK : SAMD_ECUDA; }
 
-// Largest |value| of a lane format.
-long long max_abs(samd_fmt f) { return f.is_signed ? (1LL << (f.bits - 1)) : ((1LL << f.bits) - 1); }
-
 bool shape_ok(int64_t rows, int64_t inner) { return rows >= 0 && inner >= 0 && (rows == 0 || inner <= INT64_MAX / rows); }
 
 }  // namespace
@@ -90,14 +87,14 @@ size_t samd_conv2d_workspace_size(const samd_conv_desc *d, samd_fmt fa, samd_fmt
   return conv2d_workspace_size(d, fa, fw);
 }
 
-samd_status samd_conv2d(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
-                        int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, void *workspace,
-                        size_t workspace_bytes, samd_stream_t stream) {
+namespace {
+// Checks shared by the three convolution entry points. fo.bits == 0 means no
+// packed output format.
+samd_status conv_common_checks(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fmt fo, int shift) {
   if (!d) return SAMD_EINVAL;
   if (!fmt_valid(fa) || !fmt_valid(fw)) return SAMD_EINVAL;
-  if (packed_out && !fmt_valid(fo)) return SAMD_EINVAL;
-  if (!acc_out && !packed_out) return SAMD_EINVAL;
-  if (packed_out && (shift < 0 || shift > 31)) return SAMD_EINVAL;
+  if (fo.bits != 0 && !fmt_valid(fo)) return SAMD_EINVAL;
+  if (shift < 0 || shift > 31) return SAMD_EINVAL;
   if (d->layout != SAMD_NHWC && d->layout != SAMD_NCHW) return SAMD_EINVAL;
   if (d->N < 0 || d->C < 1 || d->H < 1 || d->W < 1 || d->K < 1 || d->R < 1 || d->S < 1 || d->stride < 1 ||
       d->pad < 0)
@@ -106,9 +103,17 @@ samd_status samd_conv2d(const samd_conv_desc *d, samd_fmt fa, const void *act, s
   if (d->layout != SAMD_NHWC) return SAMD_EUNSUP;
   if (fa.spacer != 0 || fw.spacer != 0) return SAMD_EUNSUP;
   if (d->R > 16 || d->S > 16) return SAMD_EUNSUP;
-  // exactness of fp32 accumulation of integer products (every partial sum < 2^24)
-  const long long taps = static_cast<long long>(d->R) * d->S * d->C;
-  if (taps * max_abs(fa) * max_abs(fw) >= (1LL << 24)) return SAMD_EUNSUP;
+  return conv2d_check(d, fa, fw);  // exactness bound of the accumulation
+}
+}  // namespace
+
+samd_status samd_conv2d(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
+                        int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, void *workspace,
+                        size_t workspace_bytes, samd_stream_t stream) {
+  if (!acc_out && !packed_out) return SAMD_EINVAL;
+  const samd_fmt fplan = packed_out ? fo : samd_fmt{0, 0, 0, 0};
+  samd_status st = conv_common_checks(d, fa, fw, fplan, packed_out ? shift : 0);
+  if (st != SAMD_OK) return st;
   if (d->N == 0) return SAMD_OK;
   if (!act || !wt || !workspace) return SAMD_EINVAL;
   if (!aligned16(act) || !aligned16(wt) || !aligned16(workspace) || (acc_out && !aligned16(acc_out)) ||
@@ -116,6 +121,31 @@ samd_status samd_conv2d(const samd_conv_desc *d, samd_fmt fa, const void *act, s
     return SAMD_EALIGN;
   return conv2d_nhwc(d, fa, act, fw, wt, acc_out, fo, packed_out, shift, workspace, workspace_bytes,
                      reinterpret_cast<cudaStream_t>(stream));
+}
+
+samd_status samd_conv2d_prepare(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const void *wt, samd_fmt fo,
+                                void *prepared, size_t prepared_bytes, samd_stream_t stream) {
+  samd_status st = conv_common_checks(d, fa, fw, fo, 0);
+  if (st != SAMD_OK) return st;
+  if (!wt || !prepared) return SAMD_EINVAL;
+  if (!aligned16(wt) || !aligned16(prepared)) return SAMD_EALIGN;
+  return conv2d_prepare(d, fa, fw, wt, fo, prepared, prepared_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+samd_status samd_conv2d_prepared(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw,
+                                 const void *prepared, size_t prepared_bytes, int32_t *acc_out, samd_fmt fo,
+                                 void *packed_out, int shift, samd_stream_t stream) {
+  if (!acc_out && !packed_out) return SAMD_EINVAL;
+  if (packed_out && fo.bits == 0) return SAMD_EINVAL;
+  samd_status st = conv_common_checks(d, fa, fw, fo, packed_out ? shift : 0);
+  if (st != SAMD_OK) return st;
+  if (d->N == 0) return SAMD_OK;
+  if (!act || !prepared) return SAMD_EINVAL;
+  if (!aligned16(act) || !aligned16(prepared) || (acc_out && !aligned16(acc_out)) ||
+      (packed_out && !aligned16(packed_out)))
+    return SAMD_EALIGN;
+  return conv2d_run(d, fa, fw, act, prepared, prepared_bytes, acc_out, fo, packed_out, shift,
+                    reinterpret_cast<cudaStream_t>(stream));
 }
 
 samd_status samd_maxpool2x2(samd_fmt f, const void *in, void *out, int N, int C, int H, int W, samd_layout layout,

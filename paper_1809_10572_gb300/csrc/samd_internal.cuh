@@ -80,7 +80,12 @@ cudaError_t launch_elementwise(samd_op op, samd_fmt fa, const void *a, const voi
 cudaError_t launch_maxpool2x2_nhwc(samd_fmt f, const void *in, void *out, int N, int C, int H, int W,
                                    cudaStream_t s);
 
-struct ConvPlan;  // defined in conv2d.cuh
+samd_status conv2d_check(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw);
+samd_status conv2d_prepare(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const void *wt, samd_fmt fo,
+                           void *prepared, size_t prepared_bytes, cudaStream_t s);
+samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const void *act, const void *prepared,
+                       size_t prepared_bytes, int32_t *acc_out, samd_fmt fo, void *packed_out, int shift,
+                       cudaStream_t s);
 samd_status conv2d_nhwc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
                         int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, void *workspace,
                         size_t workspace_bytes, cudaStream_t s);

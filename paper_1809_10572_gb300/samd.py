@@ -43,8 +43,9 @@ SAMD_NCHW, SAMD_NHWC = 0, 1
 OPS = {"add": SAMD_ADD, "sub": SAMD_SUB, "mul": SAMD_MUL, "relu": SAMD_RELU, "requant": SAMD_REQUANT}
 
 EXPORTED = ["samd_lanes_per_word", "samd_packed_words", "samd_pack", "samd_unpack", "samd_elementwise",
-            "samd_conv2d", "samd_conv2d_workspace_size", "samd_maxpool2x2", "samd_device_status",
-            "samd_status_str", "samd_version"]
+            "samd_conv2d", "samd_conv2d_workspace_size", "samd_conv2d_prepare", "samd_conv2d_prepared",
+            "samd_maxpool2x2", "samd_device_status", "samd_status_str", "samd_version"]
+FMT_NONE = (0, 0, 0, 0)
 
 
 class SamdError(RuntimeError):
@@ -81,6 +82,11 @@ def load(build_if_missing: bool = True):
     lib.samd_conv2d.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, vp, samd_fmt, vp, vp, samd_fmt, vp, i32, vp, sz,
                                 vp]
     lib.samd_conv2d.restype = i32
+    lib.samd_conv2d_prepare.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, samd_fmt, vp, samd_fmt, vp, sz, vp]
+    lib.samd_conv2d_prepare.restype = i32
+    lib.samd_conv2d_prepared.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, vp, samd_fmt, vp, sz, vp, samd_fmt, vp,
+                                         i32, vp]
+    lib.samd_conv2d_prepared.restype = i32
     lib.samd_conv2d_workspace_size.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, samd_fmt]
     lib.samd_conv2d_workspace_size.restype = sz
     lib.samd_maxpool2x2.argtypes = [samd_fmt, vp, vp, i32, i32, i32, i32, i32, vp]
@@ -165,6 +171,25 @@ def samd_conv2d(desc, fa, act, fw, wt, acc_out, fo, packed_out, shift, workspace
     _check(load().samd_conv2d(ctypes.byref(desc), fa, _ptr(act), fw, _ptr(wt), _ptr(acc_out),
                               fo if fo is not None else samd_fmt(8, 1, 0, 32), _ptr(packed_out), shift,
                               _ptr(workspace), workspace_bytes, _stream(stream)), "samd_conv2d")
+
+
+def _nbytes(t):
+    return t.numel() * t.element_size() if isinstance(t, torch.Tensor) else 0
+
+
+def samd_conv2d_prepare(desc, fa, fw, wt, fo, prepared, prepared_bytes=None, stream=None):
+    fo = fo if fo is not None else samd_fmt(*FMT_NONE)
+    nb = _nbytes(prepared) if prepared_bytes is None else prepared_bytes
+    _check(load().samd_conv2d_prepare(ctypes.byref(desc), fa, fw, _ptr(wt), fo, _ptr(prepared), nb, _stream(stream)),
+           "samd_conv2d_prepare")
+
+
+def samd_conv2d_prepared(desc, fa, act, fw, prepared, acc_out, fo, packed_out, shift, prepared_bytes=None,
+                         stream=None):
+    fo = fo if fo is not None else samd_fmt(*FMT_NONE)
+    nb = _nbytes(prepared) if prepared_bytes is None else prepared_bytes
+    _check(load().samd_conv2d_prepared(ctypes.byref(desc), fa, _ptr(act), fw, _ptr(prepared), nb, _ptr(acc_out), fo,
+                                       _ptr(packed_out), shift, _stream(stream)), "samd_conv2d_prepared")
 
 
 def samd_maxpool2x2(f, inp, out, N, C, H, W, layout=SAMD_NHWC, stream=None):
@@ -263,6 +288,27 @@ def conv2d(act, wt, shape: ConvShape, fa: samd_fmt, fw: samd_fmt, fo: samd_fmt |
         workspace = conv_workspace(shape, fa, fw, dev)
     samd_conv2d(shape.desc(), fa, act, fw, wt, acc, fo, packed, shift, workspace, stream=stream)
     return acc, packed
+
+
+class PreparedConv:
+    """A convolution layer whose weights were widened once (samd_conv2d_prepare)."""
+
+    def __init__(self, wt_words, shape: ConvShape, fa: samd_fmt, fw: samd_fmt, fo: samd_fmt | None = None,
+                 stream=None):
+        self.shape, self.fa, self.fw, self.fo = shape, fa, fw, fo
+        self.prepared = conv_workspace(shape, fa, fw, wt_words.device)
+        samd_conv2d_prepare(shape.desc(), fa, fw, wt_words, fo, self.prepared, stream=stream)
+
+    def __call__(self, act, acc_out=None, packed_out=None, shift: int = 0, stream=None):
+        samd_conv2d_prepared(self.shape.desc(), self.fa, act, self.fw, self.prepared, acc_out, self.fo, packed_out,
+                             shift, stream=stream)
+        return acc_out, packed_out
+
+    def outputs(self, want_acc=True, want_packed=True, device="cuda"):
+        s = self.shape
+        acc = torch.empty((s.N, s.Ho, s.Wo, s.K), dtype=torch.int32, device=device) if want_acc else None
+        packed = empty_words(self.fo, s.N * s.Ho * s.Wo, s.K, device) if (want_packed and self.fo) else None
+        return acc, packed
 
 
 def maxpool2x2(words, f: samd_fmt, N: int, C: int, H: int, W: int, stream=None):

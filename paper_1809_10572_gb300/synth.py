@@ -84,9 +84,11 @@ def uniform_ints_t(seed: int, shape, lo: int, hi: int, device="cpu", offset: int
     return (v + lo).reshape(shape)
 
 
-def lanes_t(seed: int, shape, bits: int, signed: bool, device="cpu") -> torch.Tensor:
+def lanes_t(seed: int, shape, bits: int, signed: bool, device="cpu", offset: int = 0) -> torch.Tensor:
+    """Lane values for draws offset+1 .. offset+prod(shape); a slice of a large
+    input can be regenerated alone by passing its flat offset."""
     lo, hi = lane_range(bits, signed)
-    return uniform_ints_t(seed, shape, lo, hi, device)
+    return uniform_ints_t(seed, shape, lo, hi, device, offset)
 
 
 def lanes(seed: int, shape, bits: int, signed: bool) -> np.ndarray:

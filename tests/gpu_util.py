@@ -63,8 +63,30 @@ def oracle_requant_pack(acc_nhwk, shift, fo):
 
 
 def harness_shift(ba, bw, bo, k_taps):
-    """Requantize shift used for the workloads: keeps a chained activation
-    inside the output range without collapsing it to zero."""
-    import math
+    from paper_1809_10572_gb300.workloads import harness_shift as hs
 
-    return max(0, ba + bw - bo + math.ceil(math.log2(k_taps) / 2) - 2)
+    return hs(ba, bw, bo, k_taps)
+
+
+def max_abs(bits, signed):
+    return (1 << (bits - 1)) if signed else (1 << bits) - 1
+
+
+def conv_supported(shape, ba, sa, bw, sw):
+    """The exactness limits include/samd.h states for samd_conv2d."""
+    taps = shape.C * shape.R * shape.S
+    if taps * max_abs(ba, sa) * max_abs(bw, sw) < (1 << 24):
+        return True
+    return bw > 4 and taps * max_abs(ba, sa) * 16 < (1 << 24)
+
+
+def oracle_conv_rows(a_img_nhwc, w_v, shape, h0, h1):
+    """Oracle output rows [h0, h1) of one image (input given as [H][W][C]):
+    the zero padding is materialised, the needed input rows are cut out and
+    the oracle convolves them without further padding. Returns [h1-h0][Wo][K]."""
+    p, st = shape.pad, shape.stride
+    img = np.pad(a_img_nhwc, ((p, p), (p, p), (0, 0)))
+    crop = img[h0 * st:(h1 - 1) * st + shape.R]
+    out = oracle.conv2d(crop.transpose(2, 0, 1)[None], w_v.transpose(0, 3, 1, 2), stride=st, pad=0,
+                        nthreads=oracle.max_threads())
+    return out[0].transpose(1, 2, 0)

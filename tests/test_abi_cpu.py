@@ -80,10 +80,19 @@ def test_conv_argument_checks(lib):
     assert lib.samd_conv2d(ctypes.byref(nchw), fa, 16, fw, 16, 16, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_EUNSUP
     bad = samd.ConvShape(1, 16, 2, 2, 16, R=5, S=5, pad=1).desc()
     assert lib.samd_conv2d(ctypes.byref(bad), fa, 16, fw, 16, 16, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_ESHAPE
-    # u8 x u8 over 3x3x64 taps breaks the 2^24 exactness bound of fp32 accumulation
-    big = samd.ConvShape(1, 64, 8, 8, 16).desc()
-    u8 = samd.fmt(8, False)
-    assert lib.samd_conv2d(ctypes.byref(big), u8, 16, u8, 16, 16, u8, None, 0, 16, 1 << 20, None) == samd.SAMD_EUNSUP
+    # u8 x s8 over 3x3x512 taps: even split weight digits exceed 2^24 (4608 * 255 * 16)
+    big = samd.ConvShape(1, 512, 8, 8, 16).desc()
+    u8, s8, u4 = samd.fmt(8, False), samd.fmt(8, True), samd.fmt(4, False)
+    assert lib.samd_conv2d(ctypes.byref(big), u8, 16, s8, 16, 16, u8, None, 0, 16, 1 << 20, None) == samd.SAMD_EUNSUP
+    # 4-bit weights are not split: 4608 * 255 * 15 >= 2^24
+    assert lib.samd_conv2d(ctypes.byref(big), u8, 16, u4, 16, 16, u8, None, 0, 16, 1 << 20, None) == samd.SAMD_EUNSUP
+    assert lib.samd_conv2d_prepare(ctypes.byref(big), u8, s8, 16, u8, 16, 1 << 20, None) == samd.SAMD_EUNSUP
+    # the 3x3 x 64-channel u8 x u8 layer fits with split digits: rejected here only for the misaligned pointer
+    mid = samd.ConvShape(1, 64, 8, 8, 16).desc()
+    assert lib.samd_conv2d(ctypes.byref(mid), u8, 16, u8, 24, 16, u8, None, 0, 16, 1 << 20, None) == samd.SAMD_EALIGN
     assert lib.samd_conv2d(ctypes.byref(d), fa, 16, fw, 24, 16, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_EALIGN
+    assert lib.samd_conv2d_prepared(ctypes.byref(d), fa, 16, fw, 16, 1 << 20, None, fa, None, 0, None) == samd.SAMD_EINVAL
+    assert lib.samd_conv2d_prepared(ctypes.byref(d), fa, 16, fw, 16, 1 << 20, None, samd.samd_fmt(0, 0, 0, 0), 16, 0,
+                                    None) == samd.SAMD_EINVAL
     assert samd.samd_conv2d_workspace_size(d, fa, fw) > 0
     assert samd.samd_conv2d_workspace_size(samd.ConvShape(1, 0, 8, 8, 16).desc(), fa, fw) == 0

@@ -7,8 +7,8 @@ import pytest
 import torch
 
 import oracle
-from gpu_util import (assert_status_clean, conv_case, gpu_pack, harness_shift, np_words, oracle_conv_nhwc,
-                      oracle_requant_pack, values_and_bytes)
+from gpu_util import (assert_status_clean, conv_case, conv_supported, gpu_pack, harness_shift, np_words,
+                      oracle_conv_nhwc, oracle_requant_pack, values_and_bytes)
 from paper_1809_10572_gb300 import samd, synth
 
 pytestmark = pytest.mark.gpu
@@ -191,8 +191,7 @@ CONV_SHAPES = [
 @pytest.mark.parametrize("ba,sa,bw,sw", [(4, False, 4, True), (2, True, 6, False), (3, True, 3, True),
                                          (1, False, 1, True), (7, False, 5, True), (8, True, 8, True)])
 def test_conv_shapes(samd_lib, shape, ba, sa, bw, sw):
-    if shape.C * shape.R * shape.S * (1 << ba) * (1 << bw) >= (1 << 26) and ba == 8:
-        pytest.skip("beyond the single-accumulator exactness bound")
+    assert conv_supported(shape, ba, sa, bw, sw)
     run_conv_check(shape, ba, sa, bw, sw, fo_t=(ba, sa, 0, 32), seed=synth.seed_for(shape, ba, sa, bw, sw))
 
 
@@ -202,9 +201,7 @@ def test_conv_shapes(samd_lib, shape, ba, sa, bw, sw):
 @pytest.mark.parametrize("bits", BITS)
 def test_conv_every_width_and_sign(samd_lib, bits, sa, sw, word_bits):
     shape = samd.ConvShape(2, 24, 10, 9, 32)
-    if shape.C * 9 * (((1 << bits) - 1) if not sa else (1 << (bits - 1))) * \
-            (((1 << bits) - 1) if not sw else (1 << (bits - 1))) >= (1 << 24):
-        pytest.skip("beyond the single-accumulator exactness bound")
+    assert conv_supported(shape, bits, sa, bits, sw)
     run_conv_check(shape, bits, sa, bits, sw, word_bits=word_bits, fo_t=(bits, sa, 0, word_bits),
                    seed=synth.seed_for("w", bits, sa, sw, word_bits))
 
