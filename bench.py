@@ -45,6 +45,8 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--layers", type=str, default="", help="comma-separated layer indices (profiling aid)")
+    ap.add_argument("--streams", type=int, default=8,
+                    help="independent layers of a step run on this many streams (graph branches)")
     return ap.parse_args()
 
 
@@ -212,7 +214,8 @@ def workload_config(args, layers):
     return {"workload": desc, "layers": len(layers), "macs_per_step": workloads.total_macs(layers),
             "l2": "flushed before every step (512 MiB write); inputs otherwise resident in HBM",
             "weights": "prepared once into the fp16 operand layout (samd_conv2d_prepare), not in the step",
-            "launch": "one CUDA graph per step", "parallelism": f"replicas x{args.gpus}"}
+            "launch": f"one CUDA graph per step; independent layers fanned out over {args.streams} streams",
+            "parallelism": f"replicas x{args.gpus}"}
 
 
 # ---- the samd arm ------------------------------------------------------------------------
@@ -315,10 +318,17 @@ def run_samd(args, layers):
         flush_buf.fill_(1)
 
     stream = torch.cuda.Stream(device=dev)
+    side = [torch.cuda.Stream(device=dev) for _ in range(max(1, args.streams))]
 
-    def step_calls(s):
-        for b in built:
-            b["conv"](b["act"], None, b["out"], b["shift"], stream=s)
+    def step_calls(main):
+        # the layers of the workload are independent: fan them out over the
+        # side streams and join them back into `main`
+        for sd in side:
+            sd.wait_stream(main)
+        for i, b in enumerate(built):
+            b["conv"](b["act"], None, b["out"], b["shift"], stream=side[i % len(side)])
+        for sd in side:
+            main.wait_stream(sd)
 
     # first calls outside any capture (kernel attributes, tensor-map entry point)
     with torch.cuda.stream(stream):

@@ -52,6 +52,8 @@ constexpr int kThreads = 192;
 constexpr int kUnpackThreads = 128;
 constexpr uint32_t kATileBytes = BM * BK * 2;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s
+constexpr int kGatherDepth = 4;                    // packed chunks in flight per thread
+constexpr int kUnpackWarps = 4;
 
 __host__ __device__ constexpr bool pair16(int bits) { return bits == 1 || bits == 2 || bits == 4 || bits == 8; }
 
@@ -82,6 +84,7 @@ struct ConvArgs {
   int mma_n;        // MMA N: n_mma, or 2 * n_mma with split weight digits
   int split;        // 1: accumulator columns [0, n_mma) hold hi digits, [n_mma, 2 n_mma) lo digits
   int stages;
+  int gather_vec;   // AGather::vec
   uint32_t tmem_cols;
   int out_bits, out_signed, out_lane_w, out_L, out_word64, out_wpr;
   int shift;
@@ -162,15 +165,26 @@ struct AUnpack {
   }
 };
 
-// Gathers the packed words of one pixel's chunk: word kw of the reduction is
-// word (kw mod wpr) of the input pixel at tap kw / wpr; taps outside the
-// image and words past the end read zero.
+// Bytes of one pixel-chunk row in the packed staging ring (a multiple of 16).
+template <typename W, int WC>
+struct Staging {
+  static constexpr int kBytes = WC * static_cast<int>(sizeof(W));
+  static constexpr int kRowBytes = (kBytes + 15) / 16 * 16;
+  // widest cp.async that divides a whole chunk held by one pixel
+  static constexpr int kVec = kBytes % 16 == 0 ? 16 : (kBytes % 8 == 0 ? 8 : static_cast<int>(sizeof(W)));
+};
+
+// Gathers the packed words of one pixel's chunk into shared memory with
+// cp.async: word kw of the reduction is word (kw mod wpr) of the input pixel
+// at tap kw / wpr; taps outside the image and words past the end are
+// zero-filled (source size 0).
 template <typename W, int WC>
 struct AGather {
   const W *act;
   int H, W_, wpr, S, stride, pad, words_total;
   int n, oh, ow;
   bool row_valid;
+  bool vec;  // every chunk lies inside one pixel at a kVec-aligned offset
 
   __device__ __forceinline__ const W *pixel(int tap, bool &valid) const {
     int r = tap / S, s = tap - (tap / S) * S;
@@ -179,14 +193,34 @@ struct AGather {
     return act + ((static_cast<long long>(n) * H + ih) * W_ + iw) * wpr;
   }
 
-  __device__ __forceinline__ void load(int chunk, W (&dst)[WC]) const {
+  __device__ __forceinline__ void issue(int chunk, uint32_t dst) const {
+    using St = Staging<W, WC>;
     const int kw0 = chunk * WC;
     int tap = kw0 / wpr, wi = kw0 - tap * wpr;
     bool valid;
     const W *px = pixel(tap, valid);
+    if (vec) {
+      const char *src = reinterpret_cast<const char *>(valid ? px + wi : act);
+      const uint32_t nb = valid ? St::kVec : 0u;
+#pragma unroll
+      for (int v = 0; v < St::kBytes / St::kVec; ++v) {
+        if constexpr (St::kVec == 16)
+          ptx::cp_async_16(dst + 16 * v, src + 16 * v, nb);
+        else if constexpr (St::kVec == 8)
+          ptx::cp_async_8(dst + 8 * v, src + 8 * v, nb);
+        else
+          ptx::cp_async_4(dst + 4 * v, src + 4 * v, nb);
+      }
+      return;
+    }
 #pragma unroll
     for (int q = 0; q < WC; ++q) {
-      dst[q] = (valid && kw0 + q < words_total) ? __ldg(px + wi) : W(0);
+      const bool in = valid && kw0 + q < words_total;
+      const W *src = in ? px + wi : act;
+      if constexpr (sizeof(W) == 8)
+        ptx::cp_async_8(dst + 8 * q, src, in ? 8u : 0u);
+      else
+        ptx::cp_async_4(dst + 4 * q, src, in ? 4u : 0u);
       if (++wi == wpr) {
         wi = 0;
         ++tap;
@@ -206,9 +240,11 @@ __global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_const
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int ST = args.stages;
   const uint32_t b_bytes = static_cast<uint32_t>(args.mma_n) * 128u;
+  using St = Staging<W, WC>;
   uint8_t *sA = smem;
   uint8_t *sB = smem + ST * kATileBytes;
-  uint64_t *bars = reinterpret_cast<uint64_t *>(sB + ST * b_bytes);
+  uint8_t *sG = sB + ST * b_bytes;  // packed staging ring: kGatherDepth slots x 128 rows
+  uint64_t *bars = reinterpret_cast<uint64_t *>(sG + kGatherDepth * BM * St::kRowBytes);
   uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 3 * ST + 2);
   auto full_a = [&](int s) { return ptx::smem_addr(bars + s); };
   auto full_b = [&](int s) { return ptx::smem_addr(bars + ST + s); };
@@ -229,7 +265,7 @@ __global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_const
   }
   if (threadIdx.x == 32) {
     for (int s = 0; s < ST; ++s) {
-      ptx::mbar_init(full_a(s), kUnpackThreads);
+      ptx::mbar_init(full_a(s), kUnpackWarps);
       ptx::mbar_init(full_b(s), 1);
       ptx::mbar_init(empty(s), 1);
     }
@@ -316,23 +352,59 @@ __global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_const
       g.oh = static_cast<int>(t % args.Ho);
       g.n = static_cast<int>(t / args.Ho);
     }
-    W cur[WC], nxt[WC];
-    g.load(0, cur);
+    g.vec = args.gather_vec != 0;
+    const uint32_t slot0 = ptx::smem_addr(sG) + row * St::kRowBytes;
+    constexpr uint32_t kSlotBytes = BM * St::kRowBytes;
+#pragma unroll
+    for (int d = 0; d < kGatherDepth; ++d) {
+      if (d < args.nchunks) g.issue(d, slot0 + d * kSlotBytes);
+      ptx::cp_async_commit();
+    }
     for (int c = 0; c < args.nchunks; ++c) {
-      if (c + 1 < args.nchunks) g.load(c + 1, nxt);
+      const int slot = c % kGatherDepth;
+      ptx::cp_async_wait<kGatherDepth - 1>();  // this thread's copies of chunk c have landed
+      W cur[WC];
+      const uint8_t *src = sG + slot * kSlotBytes + row * St::kRowBytes;
+#pragma unroll
+      for (int v = 0; v < St::kRowBytes / 16; ++v) {
+        const uint4 t = *reinterpret_cast<const uint4 *>(src + 16 * v);
+        const uint32_t tw[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int byte = 16 * v + 4 * k;
+          if (byte < St::kBytes) {
+            if constexpr (sizeof(W) == 4) {
+              cur[byte / 4] = tw[k];
+            } else if ((k & 1) == 0) {
+              cur[byte / 8] = static_cast<W>(tw[k]) | (static_cast<W>(tw[k + 1]) << 32);
+            }
+          }
+        }
+      }
       const int s = c % ST, round = c / ST;
-      if (round > 0 && !ptx::mbar_wait_bounded(empty(s), (round - 1) & 1, status, kWaitLimitNs)) {
-        ok = false;
-        break;
+      if (round > 0) {
+        bool w_ok = true;
+        if (lane == 0) w_ok = ptx::mbar_wait_bounded(empty(s), (round - 1) & 1, status, kWaitLimitNs);
+        if (!__shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0)) {
+          ok = false;
+          break;
+        }
       }
       U::unpack_row(cur, sA + s * kATileBytes, row);
       ptx::fence_proxy_async_smem();
-      ptx::mbar_arrive(full_a(s));
-#pragma unroll
-      for (int q = 0; q < WC; ++q) cur[q] = nxt[q];
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(full_a(s));
+      // refill the slot just read (its words are in registers and consumed)
+      if (c + kGatherDepth < args.nchunks) g.issue(c + kGatherDepth, slot0 + slot * kSlotBytes);
+      ptx::cp_async_commit();
     }
+    ptx::cp_async_wait<0>();
 
-    if (ok) ok = ptx::mbar_wait_bounded(acc_bar, 0, status, kWaitLimitNs);
+    if (ok) {
+      bool w_ok = true;
+      if (lane == 0) w_ok = ptx::mbar_wait_bounded(acc_bar, 0, status, kWaitLimitNs);
+      ok = __shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0) != 0;
+    }
     // every thread of the warp must take part in tcgen05.ld
     ok = __all_sync(0xffffffffu, ok);
     if (ok) {
@@ -343,9 +415,13 @@ __global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_const
       const bool vec_ok = (args.K % 4 == 0) && (ch0 % 4 == 0);
       const int lo = lane_lo(args.out_bits, args.out_signed), hi = lane_hi(args.out_bits, args.out_signed);
       const uint32_t omask = (1u << args.out_bits) - 1;
-      uint64_t wacc = 0;
-      int wl = 0;
-      long long widx = g.row_valid && args.packed_out ? m * args.out_wpr + ch0 / args.out_L : 0;
+      // The requantized lane patterns of this row, one byte per channel, go to
+      // shared memory first (the operand ring is idle once the accumulators
+      // are complete). A row holds whole 32-channel groups plus 4 bytes: an
+      // odd number of 32-bit words, so the warp's 4-byte stores fall in
+      // distinct banks. 128 rows x (256 + 4) bytes fit in the ring.
+      const int ebytes = (args.n_mma + 31) / 32 * 32 + 4;
+      uint8_t *erow = sA + row * ebytes;
       for (int col = 0; col < nvalid; col += 32) {
         uint32_t r[32];
         int v[32];
@@ -368,33 +444,46 @@ __global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_const
             for (int i = 0; i < 8; ++i)
               reinterpret_cast<int4 *>(dst)[i] = make_int4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
           } else {
-            for (int i = 0; i < cnt; ++i) dst[i] = v[i];
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (i < cnt) dst[i] = v[i];
           }
         }
         if (args.packed_out) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            if (i < cnt) {
-              const int y = clamp_int(v[i] >> args.shift, lo, hi);
-              wacc |= static_cast<uint64_t>(static_cast<uint32_t>(y) & omask) << (wl * args.out_lane_w);
-              if (++wl == args.out_L) {
-                if (args.out_word64)
-                  static_cast<uint64_t *>(args.packed_out)[widx] = wacc;
-                else
-                  static_cast<uint32_t *>(args.packed_out)[widx] = static_cast<uint32_t>(wacc);
-                ++widx;
-                wacc = 0;
-                wl = 0;
-              }
+          for (int i4 = 0; i4 < 8; ++i4) {
+            uint32_t pk = 0;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const int y = clamp_int(v[4 * i4 + k] >> args.shift, lo, hi);
+              pk |= (static_cast<uint32_t>(y) & omask) << (8 * k);
             }
+            *reinterpret_cast<uint32_t *>(erow + col + 4 * i4) = pk;
           }
         }
       }
-      if (g.row_valid && args.packed_out && wl > 0) {
-        if (args.out_word64)
-          static_cast<uint64_t *>(args.packed_out)[widx] = wacc;
-        else
-          static_cast<uint32_t *>(args.packed_out)[widx] = static_cast<uint32_t>(wacc);
+      // each output word packs L consecutive channels of this row
+      if (g.row_valid && args.packed_out) {
+        const int Lo = args.out_L, lw = args.out_lane_w;
+        const int nwords = (nvalid + Lo - 1) / Lo;
+        const long long w0 = m * args.out_wpr + ch0 / Lo;
+        if (args.out_word64) {
+          uint64_t *dst = static_cast<uint64_t *>(args.packed_out) + w0;
+          for (int j = 0; j < nwords; ++j) {
+            const int c0 = j * Lo, cn = nvalid - c0 < Lo ? nvalid - c0 : Lo;
+            uint64_t wv = 0;
+            for (int l = 0; l < cn; ++l) wv |= static_cast<uint64_t>(erow[c0 + l]) << (l * lw);
+            dst[j] = wv;
+          }
+        } else {
+          uint32_t *dst = static_cast<uint32_t *>(args.packed_out) + w0;
+          for (int j = 0; j < nwords; ++j) {
+            const int c0 = j * Lo, cn = nvalid - c0 < Lo ? nvalid - c0 : Lo;
+            uint32_t wv = 0;
+            for (int l = 0; l < cn; ++l) wv |= static_cast<uint32_t>(erow[c0 + l]) << (l * lw);
+            dst[j] = wv;
+          }
+        }
       }
     }
   }
@@ -474,7 +563,7 @@ EncodeTiledFn encode_tiled() {
 }
 
 struct Plan {
-  int wpr, words_total, La, WC, nchunks, Kpad, NBc, n_mma, mma_n, split, nblocks, stages, Ho, Wo;
+  int wpr, words_total, La, WC, nchunks, Kpad, NBc, n_mma, mma_n, split, nblocks, stages, Ho, Wo, gather_vec;
   long long M;
   uint32_t tmem_cols;
   size_t smem_bytes;
@@ -520,12 +609,22 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
   uint32_t cols = 32;
   while (cols < static_cast<uint32_t>(p.mma_n)) cols <<= 1;
   p.tmem_cols = cols;
+  // packed staging ring: kGatherDepth slots of 128 rows x (chunk bytes rounded up to 16)
+  const int wb = fa.word_bits / 8;
+  const int chunk_bytes = p.WC * wb;
+  const size_t staging = static_cast<size_t>(kGatherDepth) * BM * ((chunk_bytes + 15) / 16 * 16);
+  const int vec = chunk_bytes % 16 == 0 ? 16 : (chunk_bytes % 8 == 0 ? 8 : wb);
+  p.gather_vec = (p.wpr % p.WC == 0) && ((static_cast<long long>(p.wpr) * wb) % vec == 0) ? 1 : 0;
   const size_t stage_bytes = kATileBytes + static_cast<size_t>(p.mma_n) * 128;
-  int st = static_cast<int>((100 * 1024) / stage_bytes);
+  const size_t fixed = 1024 + staging + 512;
+  // two CTAs per SM when at least three pipeline stages fit in half the SM's
+  // shared memory, else one CTA with a deeper ring
+  long long st = (113 * 1024 - static_cast<long long>(fixed)) / static_cast<long long>(stage_bytes);
+  if (st < 3) st = (200 * 1024 - static_cast<long long>(fixed)) / static_cast<long long>(stage_bytes);
   if (st < 2) st = 2;
   if (st > 6) st = 6;
-  p.stages = st;
-  p.smem_bytes = 1024 + st * stage_bytes + (3 * st + 2) * 8 + 16;
+  p.stages = static_cast<int>(st);
+  p.smem_bytes = fixed + p.stages * stage_bytes;
   p.ws_bytes = static_cast<size_t>(p.nblocks) * p.mma_n * p.Kpad * sizeof(__half);
   return SAMD_OK;
 }
@@ -696,6 +795,7 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   a.mma_n = p.mma_n;
   a.split = p.split;
   a.stages = p.stages;
+  a.gather_vec = p.gather_vec;
   a.tmem_cols = p.tmem_cols;
   a.out_bits = packed_out ? fo.bits : 8;
   a.out_signed = packed_out ? fo.is_signed : 1;

@@ -77,8 +77,9 @@ def test_vgg16_chain_small(samd_lib):
     """All 13 VGG-16 convolutions and the four pools chained on 32x32 inputs
     (batch 2): requantized u4 outputs feed the next layer on both sides; each
     layer's output is compared. The s4 weights are drawn from [-7, 7] so their
-    mean is zero; with the full [-8, 7] range the sums drift negative and the
-    unsigned requantize zeroes the chain after a few layers."""
+    mean is zero, and each layer's shift is calibrated on the oracle's sums
+    (their positive 99th percentile maps near the top of u4); a fixed shift
+    lets the ReLU'd signal decay to zero within a few layers."""
     layers = workloads.vgg16(N=2, H=32)
     s0 = layers[0].shape
     x = synth.lanes(synth.seed_for("chain"), (s0.N, s0.H, s0.W, s0.C), 4, False)  # NHWC values, oracle side
@@ -88,9 +89,11 @@ def test_vgg16_chain_small(samd_lib):
         s = layer.shape
         w_v = synth.uniform_ints(synth.seed_for("chainw", i), (s.K, s.R, s.S, s.C), -7, 7)
         w_w = gpu_pack(synth.to_bytes_t(torch.from_numpy(w_v)).cuda(), f4s, s.K * s.R * s.S, s.C)
-        shift = workloads.harness_shift(4, 4, 4, s.C * 9)
-        _, yw = samd.conv2d(xw, w_w, s, f4u, f4s, f4u, shift=shift, want_acc=False)
         acc = oracle_conv_nhwc(x, w_v, s)
+        pos = acc[acc > 0]
+        p99 = int(np.percentile(pos, 99)) if pos.size else 0
+        shift = max(0, p99.bit_length() - 4)
+        _, yw = samd.conv2d(xw, w_w, s, f4u, f4s, f4u, shift=shift, want_acc=False)
         y = oracle.requant(acc.ravel(), shift, 4, False).reshape(acc.shape)
         assert np.array_equal(np_words(yw, 32), oracle.pack(y.reshape(-1, s.K), 4, False)), layer.name
         assert 0 < np.count_nonzero(y) < y.size  # the chain neither saturates nor vanishes
