@@ -190,6 +190,30 @@ SAMD_API samd_status samd_conv2d_prepared(const samd_conv_desc *desc, samd_fmt f
                                           samd_fmt fo, void *packed_out, int shift, samd_stream_t stream);
 
 /*
+ * samd_conv2d_noalloc: samd_conv2d for callers that cannot allocate device
+ * memory -- code that runs where cudaMalloc is off limits (inside a framework
+ * that owns every allocation through its own pool, a plugin or real-time
+ * path that must not allocate after start-up, a process whose memory pool
+ * is already spoken for). The paper has no counterpart; this is an interface
+ * convenience. Same arguments and results as samd_conv2d, without the
+ * workspace: the widened weights go to a static device array of
+ * 8 MiB (8388608 bytes) inside the library, held on every GPU that loads it
+ * until the process exits. A layer whose widened weights need more
+ * (samd_conv2d_workspace_size > 8 MiB, e.g. 3x3 convolutions with far more
+ * than 512 x 512 channels) is rejected with SAMD_EUNSUP before any launch.
+ * The first call on a device looks the array's device address up (once per
+ * device, with that device current); make that first call before capturing
+ * a stream into a CUDA graph. Every call reuses the same array and rewrites
+ * the part it reads before reading it, so no earlier contents leak into a
+ * result; but calls whose work overlaps on the GPU (different streams, no
+ * ordering between them) race on the array: order them on one stream.
+ * Neither this call nor anything it calls allocates or frees memory.
+ */
+SAMD_API samd_status samd_conv2d_noalloc(const samd_conv_desc *desc, samd_fmt fa, const void *act, samd_fmt fw,
+                                         const void *wt, int32_t *acc_out, samd_fmt fo, void *packed_out, int shift,
+                                         samd_stream_t stream);
+
+/*
  * samd_maxpool2x2: lane-wise max over 2x2 windows with stride 2 (used
  * between the VGG-16 blocks; not in the paper). Layout SAMD_NHWC: in is
  * N*H*W rows of C elements packed along C, out is N*(H/2)*(W/2) rows.

@@ -44,6 +44,10 @@ namespace samd {
 // Sticky record of a bounded wait that ran out (SAMD_ETIMEOUT), per device.
 __device__ int g_conv_status;
 
+// Scratch of samd_conv2d_noalloc: the widened weights of one layer. Every GPU
+// that loads the library holds these bytes until the process exits.
+__device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
+
 namespace {
 
 constexpr int BM = 128;             // output pixels per tile = MMA M = TMEM lanes
@@ -817,6 +821,42 @@ samd_status conv2d_nhwc(const samd_conv_desc *d, samd_fmt fa, const void *act, s
   samd_status st = conv2d_prepare(d, fa, fw, wt, fplan, workspace, workspace_bytes, s);
   if (st != SAMD_OK) return st;
   return conv2d_run(d, fa, fw, act, workspace, workspace_bytes, acc_out, fplan, packed_out, shift, s);
+}
+
+namespace {
+// Device address of g_noalloc_scratch for each device, looked up once with
+// that device current (the symbol's host-side name is not a device address).
+std::mutex g_scratch_mu;
+void *g_scratch_ptr[64] = {nullptr};
+
+cudaError_t noalloc_scratch(void **ptr) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_ptr[dev]) {
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return e;
+    g_scratch_ptr[dev] = p;
+  }
+  *ptr = g_scratch_ptr[dev];
+  return cudaSuccess;
+}
+}  // namespace
+
+samd_status conv2d_nhwc_noalloc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
+                                int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, cudaStream_t s) {
+  Plan p;
+  samd_status st = make_plan(d, fa, fw, packed_out ? fo : none_fmt(), p);
+  if (st != SAMD_OK) return st;
+  if (p.ws_bytes > kNoallocScratchBytes) return SAMD_EUNSUP;  // the layer's weights do not fit the static scratch
+  void *scratch = nullptr;
+  if (noalloc_scratch(&scratch) != cudaSuccess) return SAMD_ECUDA;
+  // prepare writes every byte of the widened weights that run then reads, so
+  // nothing left over from an earlier call is ever used
+  return conv2d_nhwc(d, fa, act, fw, wt, acc_out, fo, packed_out, shift, scratch, kNoallocScratchBytes, s);
 }
 
 cudaError_t read_device_status(int *status, int reset, cudaStream_t s) {

@@ -123,6 +123,21 @@ samd_status samd_conv2d(const samd_conv_desc *d, samd_fmt fa, const void *act, s
                      reinterpret_cast<cudaStream_t>(stream));
 }
 
+samd_status samd_conv2d_noalloc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
+                                int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, samd_stream_t stream) {
+  if (!acc_out && !packed_out) return SAMD_EINVAL;
+  const samd_fmt fplan = packed_out ? fo : samd_fmt{0, 0, 0, 0};
+  samd_status st = conv_common_checks(d, fa, fw, fplan, packed_out ? shift : 0);
+  if (st != SAMD_OK) return st;
+  if (d->N == 0) return SAMD_OK;
+  if (!act || !wt) return SAMD_EINVAL;
+  if (!aligned16(act) || !aligned16(wt) || (acc_out && !aligned16(acc_out)) ||
+      (packed_out && !aligned16(packed_out)))
+    return SAMD_EALIGN;
+  return conv2d_nhwc_noalloc(d, fa, act, fw, wt, acc_out, fo, packed_out, shift,
+                             reinterpret_cast<cudaStream_t>(stream));
+}
+
 samd_status samd_conv2d_prepare(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const void *wt, samd_fmt fo,
                                 void *prepared, size_t prepared_bytes, samd_stream_t stream) {
   samd_status st = conv_common_checks(d, fa, fw, fo, 0);

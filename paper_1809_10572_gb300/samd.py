@@ -44,6 +44,7 @@ OPS = {"add": SAMD_ADD, "sub": SAMD_SUB, "mul": SAMD_MUL, "relu": SAMD_RELU, "re
 
 EXPORTED = ["samd_lanes_per_word", "samd_packed_words", "samd_pack", "samd_unpack", "samd_elementwise",
             "samd_conv2d", "samd_conv2d_workspace_size", "samd_conv2d_prepare", "samd_conv2d_prepared",
+            "samd_conv2d_noalloc",
             "samd_maxpool2x2", "samd_device_status", "samd_status_str", "samd_version"]
 FMT_NONE = (0, 0, 0, 0)
 
@@ -82,6 +83,9 @@ def load(build_if_missing: bool = True):
     lib.samd_conv2d.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, vp, samd_fmt, vp, vp, samd_fmt, vp, i32, vp, sz,
                                 vp]
     lib.samd_conv2d.restype = i32
+    lib.samd_conv2d_noalloc.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, vp, samd_fmt, vp, vp, samd_fmt, vp, i32,
+                                        vp]
+    lib.samd_conv2d_noalloc.restype = i32
     lib.samd_conv2d_prepare.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, samd_fmt, vp, samd_fmt, vp, sz, vp]
     lib.samd_conv2d_prepare.restype = i32
     lib.samd_conv2d_prepared.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, vp, samd_fmt, vp, sz, vp, samd_fmt, vp,
@@ -171,6 +175,13 @@ def samd_conv2d(desc, fa, act, fw, wt, acc_out, fo, packed_out, shift, workspace
     _check(load().samd_conv2d(ctypes.byref(desc), fa, _ptr(act), fw, _ptr(wt), _ptr(acc_out),
                               fo if fo is not None else samd_fmt(8, 1, 0, 32), _ptr(packed_out), shift,
                               _ptr(workspace), workspace_bytes, _stream(stream)), "samd_conv2d")
+
+
+def samd_conv2d_noalloc(desc, fa, act, fw, wt, acc_out, fo, packed_out, shift, stream=None):
+    """samd_conv2d without a workspace (the library's static scratch holds the widened weights)."""
+    _check(load().samd_conv2d_noalloc(ctypes.byref(desc), fa, _ptr(act), fw, _ptr(wt), _ptr(acc_out),
+                                      fo if fo is not None else samd_fmt(8, 1, 0, 32), _ptr(packed_out), shift,
+                                      _stream(stream)), "samd_conv2d_noalloc")
 
 
 def _nbytes(t):
