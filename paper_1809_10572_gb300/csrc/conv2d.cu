@@ -91,7 +91,12 @@ struct ConvArgs {
   int gather_vec;   // AGather::vec
   uint32_t tmem_cols;
   int out_bits, out_signed, out_lane_w, out_L, out_word64, out_wpr;
+  int out_fast;     // output lanes per word when they divide 32 (packing in registers), else 0
   int shift;
+  // halo mode (stride 1): virtual output grid of N x Hv x Wp positions
+  int Hv, Wp, HR;   // HR halo rows per tile
+  int nck;          // channel chunks per pixel (ceil(wpr / WC))
+  int taps;         // R * S
 };
 
 __device__ __forceinline__ uint32_t hsub2_bits(uint32_t a, uint32_t b) {
@@ -233,6 +238,125 @@ struct AGather {
     }
   }
 };
+
+
+// Packs 32 requantized lane patterns (zero past `cnt`) into 32 / LO words of
+// LO lanes each and stores them; LO divides 32, so every word of the
+// 32-channel group is whole.
+template <int LO, typename WO>
+__device__ __forceinline__ void pack_regs(const uint32_t (&y)[32], int lane_w, int cnt, WO *dst) {
+#pragma unroll
+  for (int k = 0; k < 32 / LO; ++k) {
+    if (k * LO < cnt) {
+      WO w = 0;
+#pragma unroll
+      for (int l = 0; l < LO; ++l) w |= static_cast<WO>(y[k * LO + l]) << (l * lane_w);
+      dst[k] = w;
+    }
+  }
+}
+
+// Epilogue of one accumulator row (one output pixel m) of channel block nb:
+// fp32 accumulators -> exact int32 -> optional int32 store, optional
+// requantize-and-pack. Called by whole warps (tcgen05.ld is collective);
+// `ebuf` is idle operand memory of at least 128 x 260 bytes.
+__device__ __forceinline__ void epilogue_row(const ConvArgs &args, uint32_t taddr, bool row_valid, long long m, int nb,
+                                             uint8_t *ebuf, int row) {
+      const int ch0 = nb * args.NBc;
+      const int nvalid = args.K - ch0 < args.NBc ? args.K - ch0 : args.NBc;
+      const bool vec_ok = (args.K % 4 == 0) && (ch0 % 4 == 0);
+      const int lo = lane_lo(args.out_bits, args.out_signed), hi = lane_hi(args.out_bits, args.out_signed);
+      const uint32_t omask = (1u << args.out_bits) - 1;
+      // The requantized lane patterns of this row, one byte per channel, go to
+      // shared memory first (the operand ring is idle once the accumulators
+      // are complete). A row holds whole 32-channel groups plus 4 bytes: an
+      // odd number of 32-bit words, so the warp's 4-byte stores fall in
+      // distinct banks. 128 rows x (256 + 4) bytes fit in the ring.
+      const int ebytes = (args.n_mma + 31) / 32 * 32 + 4;
+      uint8_t *erow = ebuf + row * ebytes;
+      for (int col = 0; col < nvalid; col += 32) {
+        uint32_t r[32];
+        int v[32];
+        ptx::tmem_ld_32x32b_x32(taddr + col, r);
+        ptx::tmem_wait_ld();
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = __float2int_rn(__uint_as_float(r[i]));
+        if (args.split) {  // acc = 16 * hi + lo
+          ptx::tmem_ld_32x32b_x32(taddr + args.n_mma + col, r);
+          ptx::tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = 16 * v[i] + __float2int_rn(__uint_as_float(r[i]));
+        }
+        if (!row_valid) continue;
+        const int cnt = nvalid - col < 32 ? nvalid - col : 32;
+        if (args.acc_out) {
+          int32_t *dst = args.acc_out + m * args.K + ch0 + col;
+          if (cnt == 32 && vec_ok) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+              reinterpret_cast<int4 *>(dst)[i] = make_int4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (i < cnt) dst[i] = v[i];
+          }
+        }
+        if (args.packed_out) {
+          uint32_t y[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            y[i] = i < cnt ? static_cast<uint32_t>(clamp_int(v[i] >> args.shift, lo, hi)) & omask : 0u;
+          if (args.out_fast) {
+            const long long w0 = m * args.out_wpr + (ch0 + col) / args.out_L;
+            const int lw = args.out_lane_w;
+            if (args.out_word64) {
+              uint64_t *dst = static_cast<uint64_t *>(args.packed_out) + w0;
+              switch (args.out_fast) {
+                case 8: pack_regs<8>(y, lw, cnt, dst); break;
+                case 16: pack_regs<16>(y, lw, cnt, dst); break;
+                default: pack_regs<32>(y, lw, cnt, dst); break;
+              }
+            } else {
+              uint32_t *dst = static_cast<uint32_t *>(args.packed_out) + w0;
+              switch (args.out_fast) {
+                case 4: pack_regs<4>(y, lw, cnt, dst); break;
+                case 8: pack_regs<8>(y, lw, cnt, dst); break;
+                case 16: pack_regs<16>(y, lw, cnt, dst); break;
+                default: pack_regs<32>(y, lw, cnt, dst); break;
+              }
+            }
+          } else {
+#pragma unroll
+            for (int i4 = 0; i4 < 8; ++i4)
+              *reinterpret_cast<uint32_t *>(erow + col + 4 * i4) =
+                  y[4 * i4] | (y[4 * i4 + 1] << 8) | (y[4 * i4 + 2] << 16) | (y[4 * i4 + 3] << 24);
+          }
+        }
+      }
+      // each output word packs L consecutive channels of this row
+      if (row_valid && args.packed_out && !args.out_fast) {
+        const int Lo = args.out_L, lw = args.out_lane_w;
+        const int nwords = (nvalid + Lo - 1) / Lo;
+        const long long w0 = m * args.out_wpr + ch0 / Lo;
+        if (args.out_word64) {
+          uint64_t *dst = static_cast<uint64_t *>(args.packed_out) + w0;
+          for (int j = 0; j < nwords; ++j) {
+            const int c0 = j * Lo, cn = nvalid - c0 < Lo ? nvalid - c0 : Lo;
+            uint64_t wv = 0;
+            for (int l = 0; l < cn; ++l) wv |= static_cast<uint64_t>(erow[c0 + l]) << (l * lw);
+            dst[j] = wv;
+          }
+        } else {
+          uint32_t *dst = static_cast<uint32_t *>(args.packed_out) + w0;
+          for (int j = 0; j < nwords; ++j) {
+            const int c0 = j * Lo, cn = nvalid - c0 < Lo ? nvalid - c0 : Lo;
+            uint32_t wv = 0;
+            for (int l = 0; l < cn; ++l) wv |= static_cast<uint32_t>(erow[c0 + l]) << (l * lw);
+            dst[j] = wv;
+          }
+        }
+      }
+}
 
 template <typename W, int BITS, bool SIGNED>
 __global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_b,
@@ -414,81 +538,250 @@ __global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_const
     if (ok) {
       ptx::tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16);
-      const int ch0 = nb * args.NBc;
-      const int nvalid = args.K - ch0 < args.NBc ? args.K - ch0 : args.NBc;
-      const bool vec_ok = (args.K % 4 == 0) && (ch0 % 4 == 0);
-      const int lo = lane_lo(args.out_bits, args.out_signed), hi = lane_hi(args.out_bits, args.out_signed);
-      const uint32_t omask = (1u << args.out_bits) - 1;
-      // The requantized lane patterns of this row, one byte per channel, go to
-      // shared memory first (the operand ring is idle once the accumulators
-      // are complete). A row holds whole 32-channel groups plus 4 bytes: an
-      // odd number of 32-bit words, so the warp's 4-byte stores fall in
-      // distinct banks. 128 rows x (256 + 4) bytes fit in the ring.
-      const int ebytes = (args.n_mma + 31) / 32 * 32 + 4;
-      uint8_t *erow = sA + row * ebytes;
-      for (int col = 0; col < nvalid; col += 32) {
-        uint32_t r[32];
-        int v[32];
-        ptx::tmem_ld_32x32b_x32(taddr + col, r);
-        ptx::tmem_wait_ld();
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] = __float2int_rn(__uint_as_float(r[i]));
-        if (args.split) {  // acc = 16 * hi + lo
-          ptx::tmem_ld_32x32b_x32(taddr + args.n_mma + col, r);
-          ptx::tmem_wait_ld();
-#pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = 16 * v[i] + __float2int_rn(__uint_as_float(r[i]));
+      epilogue_row(args, taddr, g.row_valid, m, nb, sA, row);
+    }
+  }
+
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem_base, args.tmem_cols);
+  }
+  if (!ok) atomicOr(const_cast<int *>(status), static_cast<int>(SAMD_ETIMEOUT));
+}
+
+
+// ---- halo mode: each input pixel widened once per tile ----------------------
+//
+// Stride-1 convolutions. Output positions are numbered on a virtual grid of
+// N x Hv x Wp (Hv = H + 2 pad rows and Wp = W + 2 pad columns per image);
+// rows oh < Ho and columns ow < Wo of it are real outputs, the rest are
+// computed and dropped. Position u of the same grid, read as an input, is
+// pixel (u / Wp mod Hv - pad, u mod Wp - pad) of image u / (Hv Wp), zero
+// outside the image. Output v at tap (r, s) reads input v + r Wp + s, a fixed
+// shift, so a tile of 128 consecutive v needs the HR = 128 + (R-1) Wp + S - 1
+// consecutive input rows from its first v. They are widened once into a
+// 128-byte-swizzled fp16 halo; the MMAs of tap (r, s) read halo rows
+// r Wp + s .. r Wp + s + 127 through a descriptor whose start address moves
+// by (r Wp + s) x 128 bytes. The swizzle acts on absolute address bits, so
+// any row may start a 128-row operand (base offset field 0).
+// Reduction order: channel chunk j (WC packed words of a pixel), then tap,
+// then the chunk's lane positions.
+template <typename W, int BITS, bool SIGNED>
+__global__ void __launch_bounds__(kThreads, 1) conv_halo_kernel(const __grid_constant__ CUtensorMap tmap_b,
+                                                                 const ConvArgs args) {
+  using U = AUnpack<W, BITS, SIGNED>;
+  constexpr int WC = U::WC;
+  using St = Staging<W, WC>;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ int s_skip;
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int ST = args.stages;
+  const int NHB = args.nck > 1 ? 2 : 1;
+  const uint32_t halo_bytes = static_cast<uint32_t>((args.HR + 7) / 8 * 8) * 128u;
+  const uint32_t b_bytes = static_cast<uint32_t>(args.mma_n) * 128u;
+  const uint32_t stage_g = static_cast<uint32_t>((args.HR * St::kRowBytes + 15) / 16 * 16);
+  uint8_t *sH = smem;                   // NHB halo buffers
+  uint8_t *sB = sH + NHB * halo_bytes;  // ST weight tiles
+  uint8_t *sG = sB + ST * b_bytes;      // NHB packed staging buffers, HR rows each
+  uint64_t *bars = reinterpret_cast<uint64_t *>(sG + NHB * stage_g);
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 2 * ST + 6);
+  auto full_b = [&](int s) { return ptx::smem_addr(bars + s); };
+  auto empty_b = [&](int s) { return ptx::smem_addr(bars + ST + s); };
+  auto hfull = [&](int h) { return ptx::smem_addr(bars + 2 * ST + h); };
+  auto hempty = [&](int h) { return ptx::smem_addr(bars + 2 * ST + 2 + h); };
+  const uint32_t acc_bar = ptx::smem_addr(bars + 2 * ST + 4);
+  const uint32_t drain_bar = ptx::smem_addr(bars + 2 * ST + 5);
+
+  volatile int *status = &g_conv_status;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) s_skip = *status;
+  __syncthreads();
+  if (s_skip) return;
+  if (warp == 0) {
+    ptx::tmem_alloc(ptx::smem_addr(tmem_holder), args.tmem_cols);
+    ptx::tmem_relinquish();
+  }
+  if (threadIdx.x == 32) {
+    for (int s = 0; s < ST; ++s) {
+      ptx::mbar_init(full_b(s), 1);
+      ptx::mbar_init(empty_b(s), 1);
+    }
+    for (int h = 0; h < 2; ++h) {
+      ptx::mbar_init(hfull(h), kUnpackWarps);
+      ptx::mbar_init(hempty(h), 1);
+    }
+    ptx::mbar_init(acc_bar, 1);
+    ptx::mbar_init(drain_bar, 1);
+    ptx::fence_barrier_init();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+  const int nb = blockIdx.y;
+  const int ntiles_b = args.nck * args.taps;  // weight tiles of the reduction
+  const long long v0 = static_cast<long long>(blockIdx.x) * BM;
+  const long long plane = static_cast<long long>(args.Hv) * args.Wp;
+  bool ok = true;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      ptx::prefetch_tmap(&tmap_b);
+      int issued = 0;
+      for (int c = 0; c < ntiles_b; ++c) {
+        const int s = c % ST, round = c / ST;
+        if (round > 0 && !ptx::mbar_wait_bounded(empty_b(s), (round - 1) & 1, status, kWaitLimitNs)) {
+          ok = false;
+          break;
         }
-        if (!g.row_valid) continue;
-        const int cnt = nvalid - col < 32 ? nvalid - col : 32;
-        if (args.acc_out) {
-          int32_t *dst = args.acc_out + m * args.K + ch0 + col;
-          if (cnt == 32 && vec_ok) {
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-              reinterpret_cast<int4 *>(dst)[i] = make_int4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-          } else {
-#pragma unroll
-            for (int i = 0; i < 32; ++i)
-              if (i < cnt) dst[i] = v[i];
-          }
-        }
-        if (args.packed_out) {
-#pragma unroll
-          for (int i4 = 0; i4 < 8; ++i4) {
-            uint32_t pk = 0;
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-              const int y = clamp_int(v[4 * i4 + k] >> args.shift, lo, hi);
-              pk |= (static_cast<uint32_t>(y) & omask) << (8 * k);
-            }
-            *reinterpret_cast<uint32_t *>(erow + col + 4 * i4) = pk;
-          }
-        }
+        ptx::mbar_arrive_expect_tx(full_b(s), b_bytes);
+        ptx::tma_load_2d(ptx::smem_addr(sB + s * b_bytes), &tmap_b, c * BK, nb * args.mma_n, full_b(s));
+        issued = c + 1;
       }
-      // each output word packs L consecutive channels of this row
-      if (g.row_valid && args.packed_out) {
-        const int Lo = args.out_L, lw = args.out_lane_w;
-        const int nwords = (nvalid + Lo - 1) / Lo;
-        const long long w0 = m * args.out_wpr + ch0 / Lo;
-        if (args.out_word64) {
-          uint64_t *dst = static_cast<uint64_t *>(args.packed_out) + w0;
-          for (int j = 0; j < nwords; ++j) {
-            const int c0 = j * Lo, cn = nvalid - c0 < Lo ? nvalid - c0 : Lo;
-            uint64_t wv = 0;
-            for (int l = 0; l < cn; ++l) wv |= static_cast<uint64_t>(erow[c0 + l]) << (l * lw);
-            dst[j] = wv;
+      if (!ok) {
+        for (int c = issued - ST < 0 ? 0 : issued - ST; c < issued; ++c)
+          ptx::mbar_wait_bounded(full_b(c % ST), (c / ST) & 1, status, kWaitLimitNs / 10);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = ptx::idesc_f16_f32(BM, args.mma_n);
+      for (int j = 0; j < args.nck && ok; ++j) {
+        const int hb = j % NHB;
+        if (!ptx::mbar_wait_bounded(hfull(hb), (j / NHB) & 1, status, kWaitLimitNs)) {
+          ok = false;
+          break;
+        }
+        int words = args.wpr - j * WC;
+        if (words > WC) words = WC;
+        const int ksteps = (words * U::L + 15) / 16;
+        const uint32_t hbase = ptx::smem_addr(sH + hb * halo_bytes);
+        for (int t = 0; t < args.taps; ++t) {
+          const int c = j * args.taps + t;
+          const int s = c % ST, round = c / ST;
+          if (!ptx::mbar_wait_bounded(full_b(s), round & 1, status, kWaitLimitNs)) {
+            ok = false;
+            break;
+          }
+          ptx::tc_fence_after();
+          const int r = t / args.S, sc = t - (t / args.S) * args.S;
+          const uint64_t adesc = ptx::sw128_kmajor_desc(hbase + static_cast<uint32_t>(r * args.Wp + sc) * 128u);
+          const uint64_t bdesc = ptx::sw128_kmajor_desc(ptx::smem_addr(sB + s * b_bytes));
+          for (int kk = 0; kk < ksteps; ++kk)
+            ptx::mma_f16(tmem_base, adesc + 2 * kk, bdesc + 2 * kk, idesc, (j > 0 || t > 0 || kk > 0) ? 1u : 0u);
+          ptx::mma_commit(empty_b(s));
+        }
+        ptx::mma_commit(hempty(hb));  // the halo buffer is free once these MMAs complete
+      }
+      if (ok) ptx::mma_commit(acc_bar);
+      ptx::mma_commit(drain_bar);
+      int quiet = 0;
+      ptx::mbar_wait_bounded(drain_bar, 0, &quiet, kWaitLimitNs);
+    }
+  } else {
+    const int quad = warp & 3;
+    const int t = threadIdx.x - 64;  // 0..127
+    const W *act = static_cast<const W *>(args.act);
+    const int wb = static_cast<int>(sizeof(W));
+    // cp.async the packed words of chunk j for this thread's halo rows
+    auto gather = [&](int j, int g) {
+      const uint32_t dst0 = ptx::smem_addr(sG + g * stage_g);
+      for (int hr = t; hr < args.HR; hr += kUnpackThreads) {
+        const long long u = v0 + hr;
+        const long long img = u / plane;
+        const long long rem = u - img * plane;
+        const int ih = static_cast<int>(rem / args.Wp) - args.pad;
+        const int iw = static_cast<int>(rem - (rem / args.Wp) * args.Wp) - args.pad;
+        const bool valid = img < args.N && ih >= 0 && ih < args.H && iw >= 0 && iw < args.W;
+        const W *px = act + ((img * args.H + ih) * args.W + iw) * args.wpr + j * WC;
+        const uint32_t dst = dst0 + hr * St::kRowBytes;
+        if (args.gather_vec) {
+          const char *src = reinterpret_cast<const char *>(valid ? px : act);
+          const uint32_t nbytes = valid ? St::kVec : 0u;
+#pragma unroll
+          for (int v = 0; v < St::kBytes / St::kVec; ++v) {
+            if constexpr (St::kVec == 16)
+              ptx::cp_async_16(dst + 16 * v, src + 16 * v, nbytes);
+            else if constexpr (St::kVec == 8)
+              ptx::cp_async_8(dst + 8 * v, src + 8 * v, nbytes);
+            else
+              ptx::cp_async_4(dst + 4 * v, src + 4 * v, nbytes);
           }
         } else {
-          uint32_t *dst = static_cast<uint32_t *>(args.packed_out) + w0;
-          for (int j = 0; j < nwords; ++j) {
-            const int c0 = j * Lo, cn = nvalid - c0 < Lo ? nvalid - c0 : Lo;
-            uint32_t wv = 0;
-            for (int l = 0; l < cn; ++l) wv |= static_cast<uint32_t>(erow[c0 + l]) << (l * lw);
-            dst[j] = wv;
+#pragma unroll
+          for (int q = 0; q < WC; ++q) {
+            const bool in = valid && j * WC + q < args.wpr;
+            const W *src = in ? px + q : act;
+            if constexpr (sizeof(W) == 8)
+              ptx::cp_async_8(dst + 8 * q, src, in ? 8u : 0u);
+            else
+              ptx::cp_async_4(dst + 4 * q, src, in ? 4u : 0u);
           }
         }
       }
+      (void)wb;
+    };
+    gather(0, 0);
+    ptx::cp_async_commit();
+    for (int j = 0; j < args.nck; ++j) {
+      if (j + 1 < args.nck) gather(j + 1, (j + 1) % NHB);
+      ptx::cp_async_commit();
+      ptx::cp_async_wait<1>();  // chunk j of this thread's rows has landed
+      const int hb = j % NHB;
+      if (j >= NHB) {
+        bool w_ok = true;
+        if (lane == 0) w_ok = ptx::mbar_wait_bounded(hempty(hb), ((j / NHB) - 1) & 1, status, kWaitLimitNs);
+        if (!__shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0)) {
+          ok = false;
+          break;
+        }
+      }
+      const uint8_t *stg = sG + (j % NHB) * stage_g;
+      for (int hr = t; hr < args.HR; hr += kUnpackThreads) {
+        W cur[WC];
+        const uint8_t *src = stg + hr * St::kRowBytes;
+#pragma unroll
+        for (int v = 0; v < St::kRowBytes / 16; ++v) {
+          const uint4 q4 = *reinterpret_cast<const uint4 *>(src + 16 * v);
+          const uint32_t tw[4] = {q4.x, q4.y, q4.z, q4.w};
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const int byte = 16 * v + 4 * k;
+            if (byte < St::kBytes) {
+              if constexpr (sizeof(W) == 4) {
+                cur[byte / 4] = tw[k];
+              } else if ((k & 1) == 0) {
+                cur[byte / 8] = static_cast<W>(tw[k]) | (static_cast<W>(tw[k + 1]) << 32);
+              }
+            }
+          }
+        }
+        U::unpack_row(cur, sH + hb * halo_bytes, hr);
+      }
+      ptx::fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(hfull(hb));
+    }
+    ptx::cp_async_wait<0>();
+    if (ok) {
+      bool w_ok = true;
+      if (lane == 0) w_ok = ptx::mbar_wait_bounded(acc_bar, 0, status, kWaitLimitNs);
+      ok = __shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0) != 0;
+    }
+    ok = __all_sync(0xffffffffu, ok);
+    if (ok) {
+      ptx::tc_fence_after();
+      const int row = quad * 32 + lane;
+      const long long v = v0 + row;
+      const long long img = v / plane;
+      const long long rem = v - img * plane;
+      const int oh = static_cast<int>(rem / args.Wp), ow = static_cast<int>(rem - (rem / args.Wp) * args.Wp);
+      const bool valid = img < args.N && oh < args.Ho && ow < args.Wo;
+      const long long m = (img * args.Ho + oh) * args.Wo + ow;
+      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16);
+      epilogue_row(args, taddr, valid, m, nb, sH, row);
     }
   }
 
@@ -508,6 +801,7 @@ struct WPrepArgs {
   int bits_w, signed_w, lane_w_w, Lw, wpr_w;  // weight format
   int bits_a, La, WC, wpr_a, words_total;      // reduction order set by the activation format
   int Kpad, n_mma, mma_n, NBc, split;
+  int halo, taps;  // halo: reduction order (chunk, tap, position); else (tap-major words, position)
   long long rows_total;
 };
 
@@ -528,9 +822,17 @@ __global__ void __launch_bounds__(256) wprep_kernel(const WW *__restrict__ wt, _
     const int q = j / a.La, pos = j % a.La;
     int v = 0;
     if (r < a.NBc && k < a.K && q < a.WC) {
-      const int kw = chunk * a.WC + q;
+      int tap, wi, kw;
+      if (a.halo) {  // chunk = (channel chunk, tap)
+        tap = chunk % a.taps;
+        wi = (chunk / a.taps) * a.WC + q;
+        kw = wi < a.wpr_a ? 0 : a.words_total;  // past the pixel's last word: zero
+      } else {
+        kw = chunk * a.WC + q;
+        tap = kw / a.wpr_a;
+        wi = kw % a.wpr_a;
+      }
       if (kw < a.words_total) {
-        const int tap = kw / a.wpr_a, wi = kw % a.wpr_a;
         const int ch = wi * a.La + kpos_lane(a.bits_a, pos);
         if (ch < a.C) {
           const long long wrow = static_cast<long long>(k) * a.RS + tap;
@@ -568,6 +870,8 @@ EncodeTiledFn encode_tiled() {
 
 struct Plan {
   int wpr, words_total, La, WC, nchunks, Kpad, NBc, n_mma, mma_n, split, nblocks, stages, Ho, Wo, gather_vec;
+  int halo, Hv, Wp, HR, nck, taps;  // halo mode (see conv_halo_kernel)
+  long long grid_m;                 // CTAs along the output positions
   long long M;
   uint32_t tmem_cols;
   size_t smem_bytes;
@@ -629,6 +933,39 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
   if (st > 6) st = 6;
   p.stages = static_cast<int>(st);
   p.smem_bytes = fixed + p.stages * stage_bytes;
+  p.grid_m = (p.M + BM - 1) / BM;
+
+  // Halo mode for stride-1 convolutions with several taps, when the padded
+  // virtual grid wastes little work and the halo fits in shared memory.
+  p.halo = 0;
+  p.taps = d->R * d->S;
+  p.nck = (p.wpr + p.WC - 1) / p.WC;
+  p.Hv = d->H + 2 * d->pad;
+  p.Wp = d->W + 2 * d->pad;
+  p.HR = BM + (d->R - 1) * p.Wp + (d->S - 1);
+  if (d->stride == 1 && p.taps >= 2 && p.M > 0) {
+    const double virt = static_cast<double>(d->N) * p.Hv * p.Wp;
+    const double waste = virt / static_cast<double>(p.M);
+    const int nhb = p.nck > 1 ? 2 : 1;
+    const size_t halo_bytes = static_cast<size_t>((p.HR + 7) / 8 * 8) * 128;
+    const size_t stage_g = static_cast<size_t>((p.HR * ((chunk_bytes + 15) / 16 * 16) + 15) / 16 * 16);
+    const size_t bst = static_cast<size_t>(p.mma_n) * 128;
+    const size_t hfixed = 1024 + nhb * (halo_bytes + stage_g) + 512;
+    const int ntiles_b = p.nck * p.taps;
+    long long hst = (113 * 1024 - static_cast<long long>(hfixed)) / static_cast<long long>(bst);
+    if (hst < 4) hst = (200 * 1024 - static_cast<long long>(hfixed)) / static_cast<long long>(bst);
+    if (hst > ntiles_b) hst = ntiles_b;
+    if (hst > 16) hst = 16;
+    if (waste <= 1.16 && p.HR <= 640 && hst >= 2) {
+      p.halo = 1;
+      p.stages = static_cast<int>(hst);
+      p.smem_bytes = hfixed + p.stages * bst;
+      p.nchunks = ntiles_b;
+      p.Kpad = ntiles_b * BK;
+      p.grid_m = (static_cast<long long>(d->N) * p.Hv * p.Wp + BM - 1) / BM;
+      p.gather_vec = (p.wpr % p.WC == 0) && ((static_cast<long long>(p.wpr) * wb) % vec == 0) ? 1 : 0;
+    }
+  }
   p.ws_bytes = static_cast<size_t>(p.nblocks) * p.mma_n * p.Kpad * sizeof(__half);
   return SAMD_OK;
 }
@@ -666,7 +1003,7 @@ cudaError_t ensure_smem_attr(const void *kern, size_t smem) {
 template <typename W, int BITS, bool SIGNED>
 cudaError_t launch_conv_variant(const CUtensorMap &tmap, const ConvArgs &args, dim3 grid, size_t smem,
                                 cudaStream_t s) {
-  auto kern = conv_tc_kernel<W, BITS, SIGNED>;
+  auto kern = args.HR > 0 ? conv_halo_kernel<W, BITS, SIGNED> : conv_tc_kernel<W, BITS, SIGNED>;
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void *>(kern), smem);
   if (e != cudaSuccess) return e;
   kern<<<grid, kThreads, smem, s>>>(tmap, args);
@@ -740,6 +1077,8 @@ samd_status conv2d_prepare(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, co
   wa.mma_n = p.mma_n;
   wa.NBc = p.NBc;
   wa.split = p.split;
+  wa.halo = p.halo;
+  wa.taps = p.taps;
   wa.rows_total = static_cast<long long>(p.nblocks) * p.mma_n;
   const long long total = wa.rows_total * wa.Kpad;
   const int grid = grid_for(total, 256, sm_count() * 8);
@@ -807,8 +1146,19 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   a.out_L = packed_out ? lanes_per_word(fo) : 1;
   a.out_word64 = packed_out ? (fo.word_bits == 64) : 0;
   a.out_wpr = packed_out ? static_cast<int>(words_per_row(fo, d->K)) : 0;
+  {
+    const int Lo = a.out_L;
+    const bool fast = packed_out && (fo.word_bits == 32 ? (Lo == 4 || Lo == 8 || Lo == 16 || Lo == 32)
+                                                        : (Lo == 8 || Lo == 16 || Lo == 32));
+    a.out_fast = fast ? Lo : 0;
+  }
   a.shift = shift;
-  dim3 grid(static_cast<unsigned>((p.M + BM - 1) / BM), static_cast<unsigned>(p.nblocks));
+  a.Hv = p.Hv;
+  a.Wp = p.Wp;
+  a.HR = p.halo ? p.HR : 0;  // 0 selects the gather kernel
+  a.nck = p.nck;
+  a.taps = p.taps;
+  dim3 grid(static_cast<unsigned>(p.grid_m), static_cast<unsigned>(p.nblocks));
   cudaError_t e = fa.word_bits == 32 ? launch_conv_word<uint32_t>(fa, tmap, a, grid, p.smem_bytes, s)
                                      : launch_conv_word<uint64_t>(fa, tmap, a, grid, p.smem_bytes, s);
   return e == cudaSuccess ? SAMD_OK : SAMD_ECUDA;
