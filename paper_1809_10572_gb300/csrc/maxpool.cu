@@ -1,11 +1,13 @@
 // maxpool.cu -- lane-wise 2x2 max-pool, stride 2, on NHWC tensors packed
 // along C (used between the VGG-16 blocks; the paper has no pooling).
 //
-// One thread per output word. For spacer-free lanes the max of two words is
+// For spacer-free lanes the max of two words is
 // taken for all lanes at once: a lane-wise subtract with the MSBs as
 // temporary spacers (section 3, Fig. 5) yields each lane's borrow, i.e.
 // a < b, which selects the larger lane. Signed lanes are compared after
 // flipping their sign bits (two's complement order = offset-binary order).
+#include <cstring>
+
 #include "samd_internal.cuh"
 
 namespace samd {
@@ -34,23 +36,46 @@ __device__ __forceinline__ W swar_max(W a, W b, W flip) {
   return (b & E) | (a & ~E);
 }
 
-template <typename W, int BITS>
-__global__ void __launch_bounds__(kThreads) maxpool_swar_kernel(const W *__restrict__ in, W *__restrict__ out,
-                                                                int N, int H, int W_, int wpr, int is_signed) {
-  const int Ho = H / 2, Wo = W_ / 2;
-  const int64_t total = (int64_t)N * Ho * Wo * wpr;
+// Blocks loop over output rows (image n, row i); threads run over the row's
+// (pixel, unit) pairs, a unit being V consecutive words of a pixel (V = 4
+// 32-bit or 2 64-bit words, one 16-byte vector, when a pixel's words allow;
+// else V = 1). Index math stays in 32 bits.
+template <typename W, int BITS, int V>
+__global__ void __launch_bounds__(kThreads) maxpool_swar_kernel(const W *__restrict__ in, W *__restrict__ out, int Ho,
+                                                                int Wo, int H, int W_, int wpr, int is_signed, int rows) {
+  const int upp = wpr / V;  // units per pixel
+  const int units = Wo * upp;
   const W flip = is_signed ? PoolMasks<W, BITS>::kMsb : W(0);
-  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total; t += (int64_t)gridDim.x * blockDim.x) {
-    int64_t px = t / wpr;
-    int wi = static_cast<int>(t - px * wpr);
-    int j = static_cast<int>(px % Wo);
-    int64_t r = px / Wo;
-    int i = static_cast<int>(r % Ho);
-    int64_t n = r / Ho;
-    int64_t base = ((n * H + 2 * i) * W_ + 2 * j) * wpr + wi;
-    W m = swar_max<W, BITS>(__ldg(in + base), __ldg(in + base + wpr), flip);
-    W m2 = swar_max<W, BITS>(__ldg(in + base + (int64_t)W_ * wpr), __ldg(in + base + (int64_t)W_ * wpr + wpr), flip);
-    out[t] = swar_max<W, BITS>(m, m2, flip);
+  for (int row = blockIdx.x; row < rows; row += gridDim.x) {  // row = n * Ho + i
+  const int n = row / Ho, i = row - (row / Ho) * Ho;
+  const W *top = in + (static_cast<long long>(n) * H + 2 * i) * W_ * wpr;
+  const W *bot = top + static_cast<long long>(W_) * wpr;
+  W *dst = out + static_cast<long long>(row) * Wo * wpr;
+  for (int u = blockIdx.y * blockDim.x + threadIdx.x; u < units; u += gridDim.y * blockDim.x) {
+    const int j = u / upp, q = u - (u / upp) * upp;
+    const int off = 2 * j * wpr + q * V;
+    if constexpr (V == 1) {
+      const W m1 = swar_max<W, BITS>(__ldcs(top + off), __ldcs(top + off + wpr), flip);
+      const W m2 = swar_max<W, BITS>(__ldcs(bot + off), __ldcs(bot + off + wpr), flip);
+      dst[j * wpr + q] = swar_max<W, BITS>(m1, m2, flip);
+    } else {
+      const uint4 a = __ldcs(reinterpret_cast<const uint4 *>(top + off));
+      const uint4 b = __ldcs(reinterpret_cast<const uint4 *>(top + off + wpr));
+      const uint4 c = __ldcs(reinterpret_cast<const uint4 *>(bot + off));
+      const uint4 d = __ldcs(reinterpret_cast<const uint4 *>(bot + off + wpr));
+      W wa[V], wbv[V], wc[V], wd[V], wo[V];
+      memcpy(wa, &a, 16);
+      memcpy(wbv, &b, 16);
+      memcpy(wc, &c, 16);
+      memcpy(wd, &d, 16);
+#pragma unroll
+      for (int k = 0; k < V; ++k)
+        wo[k] = swar_max<W, BITS>(swar_max<W, BITS>(wa[k], wbv[k], flip), swar_max<W, BITS>(wc[k], wd[k], flip), flip);
+      uint4 o;
+      memcpy(&o, wo, 16);
+      __stcs(reinterpret_cast<uint4 *>(dst + j * wpr + q * V), o);
+    }
+  }
   }
 }
 
@@ -95,10 +120,25 @@ cudaError_t pool_dispatch(samd_fmt f, const void *in, void *out, int N, int C, i
                                                      lanes_per_word(f));
     return cudaGetLastError();
   }
-  switch (f.bits) {
-#define SAMD_POOL_CASE(B) \
-  case B:                 \
-    maxpool_swar_kernel<W, B><<<grid, kThreads, 0, s>>>(pi, po, N, H, W_, wpr, f.is_signed); \
+  const int Ho = H / 2, Wo = W_ / 2;
+  constexpr int V16 = 16 / static_cast<int>(sizeof(W));
+  const bool vec = (wpr % V16) == 0;
+  const int units = Wo * (vec ? wpr / V16 : wpr);
+  int gy = (units + kThreads - 1) / kThreads;
+  if (gy > 65535) gy = 65535;
+  if (static_cast<long long>(N) * Ho > 2147483647LL) return cudaErrorInvalidValue;
+  const int rows = N * Ho;
+  // enough blocks to fill the GPU (8 per SM), each looping over rows
+  long long gx = (static_cast<long long>(sm_count()) * 8 + gy - 1) / gy;
+  if (gx > rows) gx = rows;
+  const dim3 pgrid(static_cast<unsigned>(gx), gy);
+  switch (f.bits * 2 + (vec ? 1 : 0)) {
+#define SAMD_POOL_CASE(B)                                                                                   \
+  case 2 * B:                                                                                               \
+    maxpool_swar_kernel<W, B, 1><<<pgrid, kThreads, 0, s>>>(pi, po, Ho, Wo, H, W_, wpr, f.is_signed, rows); \
+    break;                                                                                                  \
+  case 2 * B + 1:                                                                                           \
+    maxpool_swar_kernel<W, B, V16><<<pgrid, kThreads, 0, s>>>(pi, po, Ho, Wo, H, W_, wpr, f.is_signed, rows); \
     break;
     SAMD_POOL_CASE(1) SAMD_POOL_CASE(2) SAMD_POOL_CASE(3) SAMD_POOL_CASE(4)
     SAMD_POOL_CASE(5) SAMD_POOL_CASE(6) SAMD_POOL_CASE(7) SAMD_POOL_CASE(8)
