@@ -34,6 +34,7 @@
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
 
+#include <cstring>
 #include <mutex>
 
 #include "samd_internal.cuh"
@@ -52,7 +53,6 @@ namespace {
 
 constexpr int BM = 128;             // output pixels per tile = MMA M = TMEM lanes
 constexpr int BK = 64;              // fp16 reduction elements per chunk = one 128-byte row
-constexpr int kThreads = 192;
 constexpr int kUnpackThreads = 128;
 constexpr uint32_t kATileBytes = BM * BK * 2;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s
@@ -74,6 +74,23 @@ __host__ __device__ constexpr int kpos_lane(int bits, int pos) {
   return pos;
 }
 
+// n / d for 0 <= n < 2^31 by one multiply-high, an add and a shift:
+// l = ceil(log2 d), m = floor(2^32 (2^l - d) / d) + 1, q = (umulhi(m, n) + n) >> l.
+struct FastDiv {
+  uint32_t m;
+  int l;
+  uint32_t d;
+};
+
+inline FastDiv make_fastdiv(uint32_t d) {
+  int l = 0;
+  while ((uint64_t(1) << l) < d) ++l;
+  const uint64_t m = ((uint64_t(1) << 32) * ((uint64_t(1) << l) - d)) / d + 1;
+  return FastDiv{static_cast<uint32_t>(m), l, d};
+}
+
+__device__ __forceinline__ uint32_t fdiv(uint32_t n, const FastDiv &f) { return (__umulhi(f.m, n) + n) >> f.l; }
+
 struct ConvArgs {
   const void *act;
   int32_t *acc_out;
@@ -87,7 +104,11 @@ struct ConvArgs {
   int n_mma;        // NBc rounded up to 16
   int mma_n;        // MMA N: n_mma, or 2 * n_mma with split weight digits
   int split;        // 1: accumulator columns [0, n_mma) hold hi digits, [n_mma, 2 n_mma) lo digits
-  int stages;
+  int stages;       // weight tiles in flight (or resident)
+  int stages_a;     // GATHER: A tiles in flight
+  int b_resident;   // 1: all weight tiles of the layer stay in shared memory
+  long long grid_m; // 128-position tiles along the output
+  int nblocks;      // channel blocks
   int gather_vec;   // AGather::vec
   uint32_t tmem_cols;
   int out_bits, out_signed, out_lane_w, out_L, out_word64, out_wpr;
@@ -97,6 +118,9 @@ struct ConvArgs {
   int Hv, Wp, HR;   // HR halo rows per tile
   int nck;          // channel chunks per pixel (ceil(wpr / WC))
   int taps;         // R * S
+  FastDiv fd_plane, fd_wp;  // halo: / (Hv * Wp), / Wp
+  FastDiv fd_wo, fd_ho;     // output pixel index -> (n, oh, ow)
+  FastDiv fd_gm;            // tile -> (channel block, position tile)
 };
 
 __device__ __forceinline__ uint32_t hsub2_bits(uint32_t a, uint32_t b) {
@@ -245,14 +269,26 @@ struct AGather {
 // 32-channel group is whole.
 template <int LO, typename WO>
 __device__ __forceinline__ void pack_regs(const uint32_t (&y)[32], int lane_w, int cnt, WO *dst) {
+  constexpr int NW = 32 / LO;  // words of this 32-channel group
+  WO w[NW];
 #pragma unroll
-  for (int k = 0; k < 32 / LO; ++k) {
-    if (k * LO < cnt) {
-      WO w = 0;
+  for (int k = 0; k < NW; ++k) {
+    w[k] = 0;
 #pragma unroll
-      for (int l = 0; l < LO; ++l) w |= static_cast<WO>(y[k * LO + l]) << (l * lane_w);
-      dst[k] = w;
+    for (int l = 0; l < LO; ++l) w[k] |= static_cast<WO>(y[k * LO + l]) << (l * lane_w);
+  }
+  constexpr int kWordBytes = static_cast<int>(sizeof(WO));
+  if (cnt == 32 && (NW * kWordBytes) % 16 == 0 && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+#pragma unroll
+    for (int v = 0; v < NW * kWordBytes / 16; ++v) {
+      uint4 q;
+      memcpy(&q, reinterpret_cast<const uint8_t *>(w) + 16 * v, 16);
+      reinterpret_cast<uint4 *>(dst)[v] = q;
     }
+  } else {
+#pragma unroll
+    for (int k = 0; k < NW; ++k)
+      if (k * LO < cnt) dst[k] = w[k];
   }
 }
 
@@ -358,200 +394,6 @@ __device__ __forceinline__ void epilogue_row(const ConvArgs &args, uint32_t tadd
       }
 }
 
-template <typename W, int BITS, bool SIGNED>
-__global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_constant__ CUtensorMap tmap_b,
-                                                               const ConvArgs args) {
-  using U = AUnpack<W, BITS, SIGNED>;
-  constexpr int WC = U::WC;
-  extern __shared__ uint8_t smem_raw[];
-  __shared__ int s_skip;
-  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const int ST = args.stages;
-  const uint32_t b_bytes = static_cast<uint32_t>(args.mma_n) * 128u;
-  using St = Staging<W, WC>;
-  uint8_t *sA = smem;
-  uint8_t *sB = smem + ST * kATileBytes;
-  uint8_t *sG = sB + ST * b_bytes;  // packed staging ring: kGatherDepth slots x 128 rows
-  uint64_t *bars = reinterpret_cast<uint64_t *>(sG + kGatherDepth * BM * St::kRowBytes);
-  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 3 * ST + 2);
-  auto full_a = [&](int s) { return ptx::smem_addr(bars + s); };
-  auto full_b = [&](int s) { return ptx::smem_addr(bars + ST + s); };
-  auto empty = [&](int s) { return ptx::smem_addr(bars + 2 * ST + s); };
-  const uint32_t acc_bar = ptx::smem_addr(bars + 3 * ST);
-  const uint32_t drain_bar = ptx::smem_addr(bars + 3 * ST + 1);
-
-  volatile int *status = &g_conv_status;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-  if (threadIdx.x == 0) s_skip = *status;  // an earlier failure: leave the outputs alone
-  __syncthreads();
-  if (s_skip) return;
-
-  if (warp == 0) {
-    ptx::tmem_alloc(ptx::smem_addr(tmem_holder), args.tmem_cols);
-    ptx::tmem_relinquish();
-  }
-  if (threadIdx.x == 32) {
-    for (int s = 0; s < ST; ++s) {
-      ptx::mbar_init(full_a(s), kUnpackWarps);
-      ptx::mbar_init(full_b(s), 1);
-      ptx::mbar_init(empty(s), 1);
-    }
-    ptx::mbar_init(acc_bar, 1);
-    ptx::mbar_init(drain_bar, 1);
-    ptx::fence_barrier_init();
-  }
-  ptx::tc_fence_before();
-  __syncthreads();
-  ptx::tc_fence_after();
-  const uint32_t tmem_base = *tmem_holder;
-
-  const int nb = blockIdx.y;
-  bool ok = true;
-
-  if (warp == 0) {
-    if (lane == 0) {
-      // ---- weight tiles by TMA ----
-      ptx::prefetch_tmap(&tmap_b);
-      int issued = 0;
-      for (int c = 0; c < args.nchunks; ++c) {
-        const int s = c % ST, round = c / ST;
-        if (round > 0 && !ptx::mbar_wait_bounded(empty(s), (round - 1) & 1, status, kWaitLimitNs)) {
-          ok = false;
-          break;
-        }
-        ptx::mbar_arrive_expect_tx(full_b(s), b_bytes);
-        ptx::tma_load_2d(ptx::smem_addr(sB + s * b_bytes), &tmap_b, c * BK, nb * args.mma_n, full_b(s));
-        issued = c + 1;
-      }
-      if (!ok) {
-        // do not leave copies in flight into shared memory: wait (bounded) for
-        // the ones whose completion nobody observed
-        for (int c = issued - ST < 0 ? 0 : issued - ST; c < issued; ++c)
-          ptx::mbar_wait_bounded(full_b(c % ST), (c / ST) & 1, status, kWaitLimitNs / 10);
-      }
-    }
-  } else if (warp == 1) {
-    if (lane == 0) {
-      // ---- MMA issue ----
-      const uint32_t idesc = ptx::idesc_f16_f32(BM, args.mma_n);
-      for (int c = 0; c < args.nchunks; ++c) {
-        const int s = c % ST, round = c / ST;
-        if (!ptx::mbar_wait_bounded(full_a(s), round & 1, status, kWaitLimitNs) ||
-            !ptx::mbar_wait_bounded(full_b(s), round & 1, status, kWaitLimitNs)) {
-          ok = false;
-          break;
-        }
-        ptx::tc_fence_after();
-        const uint64_t adesc = ptx::sw128_kmajor_desc(ptx::smem_addr(sA + s * kATileBytes));
-        const uint64_t bdesc = ptx::sw128_kmajor_desc(ptx::smem_addr(sB + s * b_bytes));
-        int words = args.words_total - c * WC;
-        if (words > WC) words = WC;
-        const int ksteps = (words * U::L + 15) / 16;
-        for (int kk = 0; kk < ksteps; ++kk)
-          ptx::mma_f16(tmem_base, adesc + 2 * kk, bdesc + 2 * kk, idesc, (c > 0 || kk > 0) ? 1u : 0u);
-        ptx::mma_commit(empty(s));
-      }
-      if (ok) ptx::mma_commit(acc_bar);
-      // all MMAs of this CTA must be complete before TMEM is released
-      ptx::mma_commit(drain_bar);
-      int quiet = 0;
-      ptx::mbar_wait_bounded(drain_bar, 0, &quiet, kWaitLimitNs);
-    }
-  } else {
-    // ---- activation gather + widen, then the epilogue ----
-    const int quad = warp & 3;  // TMEM lanes 32*quad .. 32*quad+31 belong to this warp
-    const int row = quad * 32 + lane;
-    const long long m = static_cast<long long>(blockIdx.x) * BM + row;
-    AGather<W, WC> g;
-    g.act = static_cast<const W *>(args.act);
-    g.H = args.H;
-    g.W_ = args.W;
-    g.wpr = args.wpr;
-    g.S = args.S;
-    g.stride = args.stride;
-    g.pad = args.pad;
-    g.words_total = args.words_total;
-    g.row_valid = m < args.M;
-    {
-      const long long mm = g.row_valid ? m : 0;
-      g.ow = static_cast<int>(mm % args.Wo);
-      const long long t = mm / args.Wo;
-      g.oh = static_cast<int>(t % args.Ho);
-      g.n = static_cast<int>(t / args.Ho);
-    }
-    g.vec = args.gather_vec != 0;
-    const uint32_t slot0 = ptx::smem_addr(sG) + row * St::kRowBytes;
-    constexpr uint32_t kSlotBytes = BM * St::kRowBytes;
-#pragma unroll
-    for (int d = 0; d < kGatherDepth; ++d) {
-      if (d < args.nchunks) g.issue(d, slot0 + d * kSlotBytes);
-      ptx::cp_async_commit();
-    }
-    for (int c = 0; c < args.nchunks; ++c) {
-      const int slot = c % kGatherDepth;
-      ptx::cp_async_wait<kGatherDepth - 1>();  // this thread's copies of chunk c have landed
-      W cur[WC];
-      const uint8_t *src = sG + slot * kSlotBytes + row * St::kRowBytes;
-#pragma unroll
-      for (int v = 0; v < St::kRowBytes / 16; ++v) {
-        const uint4 t = *reinterpret_cast<const uint4 *>(src + 16 * v);
-        const uint32_t tw[4] = {t.x, t.y, t.z, t.w};
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const int byte = 16 * v + 4 * k;
-          if (byte < St::kBytes) {
-            if constexpr (sizeof(W) == 4) {
-              cur[byte / 4] = tw[k];
-            } else if ((k & 1) == 0) {
-              cur[byte / 8] = static_cast<W>(tw[k]) | (static_cast<W>(tw[k + 1]) << 32);
-            }
-          }
-        }
-      }
-      const int s = c % ST, round = c / ST;
-      if (round > 0) {
-        bool w_ok = true;
-        if (lane == 0) w_ok = ptx::mbar_wait_bounded(empty(s), (round - 1) & 1, status, kWaitLimitNs);
-        if (!__shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0)) {
-          ok = false;
-          break;
-        }
-      }
-      U::unpack_row(cur, sA + s * kATileBytes, row);
-      ptx::fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(full_a(s));
-      // refill the slot just read (its words are in registers and consumed)
-      if (c + kGatherDepth < args.nchunks) g.issue(c + kGatherDepth, slot0 + slot * kSlotBytes);
-      ptx::cp_async_commit();
-    }
-    ptx::cp_async_wait<0>();
-
-    if (ok) {
-      bool w_ok = true;
-      if (lane == 0) w_ok = ptx::mbar_wait_bounded(acc_bar, 0, status, kWaitLimitNs);
-      ok = __shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0) != 0;
-    }
-    // every thread of the warp must take part in tcgen05.ld
-    ok = __all_sync(0xffffffffu, ok);
-    if (ok) {
-      ptx::tc_fence_after();
-      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16);
-      epilogue_row(args, taddr, g.row_valid, m, nb, sA, row);
-    }
-  }
-
-  ptx::tc_fence_before();
-  __syncthreads();
-  if (warp == 0) {
-    ptx::tc_fence_after();
-    ptx::tmem_dealloc(tmem_base, args.tmem_cols);
-  }
-  if (!ok) atomicOr(const_cast<int *>(status), static_cast<int>(SAMD_ETIMEOUT));
-}
-
-
 // ---- halo mode: each input pixel widened once per tile ----------------------
 //
 // Stride-1 convolutions. Output positions are numbered on a virtual grid of
@@ -568,31 +410,95 @@ __global__ void __launch_bounds__(kThreads, 2) conv_tc_kernel(const __grid_const
 // any row may start a 128-row operand (base offset field 0).
 // Reduction order: channel chunk j (WC packed words of a pixel), then tap,
 // then the chunk's lane positions.
-template <typename W, int BITS, bool SIGNED>
-__global__ void __launch_bounds__(kThreads, 1) conv_halo_kernel(const __grid_constant__ CUtensorMap tmap_b,
-                                                                 const ConvArgs args) {
+// Issues `ksteps` (1..4) MMAs of K = 16 as straight-line code: an issuing
+// loop between them measurably slows the tensor core's intake.
+__device__ __forceinline__ void mma_ksteps(int ksteps, uint32_t d, uint64_t a, uint64_t b, uint32_t idesc,
+                                           uint32_t acc) {
+  switch (ksteps) {
+    case 4:
+      ptx::mma_f16(d, a, b, idesc, acc);
+      ptx::mma_f16(d, a + 2, b + 2, idesc, 1u);
+      ptx::mma_f16(d, a + 4, b + 4, idesc, 1u);
+      ptx::mma_f16(d, a + 6, b + 6, idesc, 1u);
+      break;
+    case 3:
+      ptx::mma_f16(d, a, b, idesc, acc);
+      ptx::mma_f16(d, a + 2, b + 2, idesc, 1u);
+      ptx::mma_f16(d, a + 4, b + 4, idesc, 1u);
+      break;
+    case 2:
+      ptx::mma_f16(d, a, b, idesc, acc);
+      ptx::mma_f16(d, a + 2, b + 2, idesc, 1u);
+      break;
+    default:
+      ptx::mma_f16(d, a, b, idesc, acc);
+      break;
+  }
+}
+
+// ---- the persistent convolution kernel ----------------------------------------
+//
+// One CTA per SM loops over output tiles (tile = blockIdx.x + i * gridDim.x;
+// tile = nb * grid_m + mt: channel block nb, 128-position tile mt). Ten warps
+// with fixed roles, connected by mbarrier rings:
+//   warp 0      TMEM allocation; lane 0 streams weight tiles with TMA. When
+//               the layer has one channel block and all its weight tiles fit,
+//               they are loaded once and stay resident.
+//   warp 1      lane 0 issues tcgen05.mma into one of two TMEM accumulators,
+//               so tile i+1 accumulates while the epilogue drains tile i.
+//   warps 2-5   operand producers.
+//               HALO: for each (tile, channel chunk) the HR input rows the tile
+//               needs are gathered with cp.async and widened once into one of
+//               two fp16 halo buffers; every tap reads the halo through a
+//               descriptor shifted by r*Wp + s rows (see the halo notes above).
+//               GATHER: for each (tile, chunk) each thread gathers its pixel's
+//               packed words (implicit im2col, zero padding) through a
+//               cp.async ring and widens them into a ring of A tiles.
+//   warps 6-9   epilogue: tcgen05.ld, exact int32, optional int32 store,
+//               optional requantize-and-pack (warp w reads TMEM lanes of
+//               quadrant w % 4).
+// Every wait is bounded; a role that gives up records SAMD_ETIMEOUT and stops.
+constexpr int kPThreads = 320;
+
+template <typename W, int BITS, bool SIGNED, bool HALO>
+__global__ void __launch_bounds__(kPThreads, 1) conv_persistent_kernel(const __grid_constant__ CUtensorMap tmap_b,
+                                                                       const ConvArgs args) {
   using U = AUnpack<W, BITS, SIGNED>;
   constexpr int WC = U::WC;
   using St = Staging<W, WC>;
   extern __shared__ uint8_t smem_raw[];
   __shared__ int s_skip;
+  __shared__ uint32_t s_aoff[256];  // HALO: byte offset of tap t's first halo row
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const int ST = args.stages;
-  const int NHB = args.nck > 1 ? 2 : 1;
-  const uint32_t halo_bytes = static_cast<uint32_t>((args.HR + 7) / 8 * 8) * 128u;
+
+  const int STA = args.stages_a;  // GATHER: A tiles in flight
+  const int STB = args.stages;    // weight tiles in flight (or resident)
+  const bool resident = args.b_resident != 0;
   const uint32_t b_bytes = static_cast<uint32_t>(args.mma_n) * 128u;
+  const uint32_t halo_bytes = static_cast<uint32_t>((args.HR + 7) / 8 * 8) * 128u;
   const uint32_t stage_g = static_cast<uint32_t>((args.HR * St::kRowBytes + 15) / 16 * 16);
-  uint8_t *sH = smem;                   // NHB halo buffers
-  uint8_t *sB = sH + NHB * halo_bytes;  // ST weight tiles
-  uint8_t *sG = sB + ST * b_bytes;      // NHB packed staging buffers, HR rows each
-  uint64_t *bars = reinterpret_cast<uint64_t *>(sG + NHB * stage_g);
-  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 2 * ST + 6);
+  constexpr uint32_t kSlotBytes = BM * St::kRowBytes;  // GATHER staging slot
+
+  // shared memory carve-up (the host sizes the same regions)
+  uint8_t *sOp = smem;  // HALO: 2 halo buffers; GATHER: STA A tiles
+  const uint32_t op_bytes = HALO ? 2 * halo_bytes : STA * kATileBytes;
+  uint8_t *sB = sOp + op_bytes;
+  uint8_t *sG = sB + STB * b_bytes;  // packed staging
+  const uint32_t g_bytes = HALO ? 2 * stage_g : kGatherDepth * kSlotBytes;
+  uint8_t *sE = sG + g_bytes;  // epilogue byte rows (only for output words the registers cannot pack)
+  const uint32_t e_bytes = args.out_fast || !args.packed_out ? 0u
+                                                             : static_cast<uint32_t>(BM * ((args.n_mma + 31) / 32 * 32 + 4));
+  uint64_t *bars = reinterpret_cast<uint64_t *>(sE + (e_bytes + 15) / 16 * 16);
+  // barriers: full_b[STB] empty_b[STB] opfull[NO] opempty[NO] accfull[2] accempty[2] drain
+  const int NO = HALO ? 2 : STA;
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 2 * STB + 2 * NO + 5);
   auto full_b = [&](int s) { return ptx::smem_addr(bars + s); };
-  auto empty_b = [&](int s) { return ptx::smem_addr(bars + ST + s); };
-  auto hfull = [&](int h) { return ptx::smem_addr(bars + 2 * ST + h); };
-  auto hempty = [&](int h) { return ptx::smem_addr(bars + 2 * ST + 2 + h); };
-  const uint32_t acc_bar = ptx::smem_addr(bars + 2 * ST + 4);
-  const uint32_t drain_bar = ptx::smem_addr(bars + 2 * ST + 5);
+  auto empty_b = [&](int s) { return ptx::smem_addr(bars + STB + s); };
+  auto opfull = [&](int s) { return ptx::smem_addr(bars + 2 * STB + s); };
+  auto opempty = [&](int s) { return ptx::smem_addr(bars + 2 * STB + NO + s); };
+  auto accfull = [&](int a) { return ptx::smem_addr(bars + 2 * STB + 2 * NO + a); };
+  auto accempty = [&](int a) { return ptx::smem_addr(bars + 2 * STB + 2 * NO + 2 + a); };
+  const uint32_t drain_bar = ptx::smem_addr(bars + 2 * STB + 2 * NO + 4);
 
   volatile int *status = &g_conv_status;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -604,184 +510,368 @@ __global__ void __launch_bounds__(kThreads, 1) conv_halo_kernel(const __grid_con
     ptx::tmem_relinquish();
   }
   if (threadIdx.x == 32) {
-    for (int s = 0; s < ST; ++s) {
+    for (int s = 0; s < STB; ++s) {
       ptx::mbar_init(full_b(s), 1);
       ptx::mbar_init(empty_b(s), 1);
     }
-    for (int h = 0; h < 2; ++h) {
-      ptx::mbar_init(hfull(h), kUnpackWarps);
-      ptx::mbar_init(hempty(h), 1);
+    for (int s = 0; s < NO; ++s) {
+      ptx::mbar_init(opfull(s), kUnpackWarps);
+      ptx::mbar_init(opempty(s), 1);
     }
-    ptx::mbar_init(acc_bar, 1);
+    for (int a = 0; a < 2; ++a) {
+      ptx::mbar_init(accfull(a), 1);
+      ptx::mbar_init(accempty(a), kUnpackWarps);  // the four epilogue warps
+    }
     ptx::mbar_init(drain_bar, 1);
     ptx::fence_barrier_init();
+    if (HALO)
+      for (int t = 0; t < args.taps && t < 256; ++t)
+        s_aoff[t] = static_cast<uint32_t>((t / args.S) * args.Wp + t % args.S) * 128u;
   }
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
-  const int nb = blockIdx.y;
-  const int ntiles_b = args.nck * args.taps;  // weight tiles of the reduction
-  const long long v0 = static_cast<long long>(blockIdx.x) * BM;
-  const long long plane = static_cast<long long>(args.Hv) * args.Wp;
+
+  const long long total_tiles = static_cast<long long>(args.grid_m) * args.nblocks;
+  const long long first_tile = blockIdx.x, tile_step = gridDim.x;
+  const int nchunks = args.nchunks;  // weight tiles per output tile
   bool ok = true;
 
   if (warp == 0) {
     if (lane == 0) {
+      // ---- weight tiles ----
       ptx::prefetch_tmap(&tmap_b);
-      int issued = 0;
-      for (int c = 0; c < ntiles_b; ++c) {
-        const int s = c % ST, round = c / ST;
-        if (round > 0 && !ptx::mbar_wait_bounded(empty_b(s), (round - 1) & 1, status, kWaitLimitNs)) {
-          ok = false;
-          break;
+      if (resident) {
+        for (int c = 0; c < nchunks; ++c) {
+          ptx::mbar_arrive_expect_tx(full_b(c), b_bytes);
+          ptx::tma_load_2d(ptx::smem_addr(sB + c * b_bytes), &tmap_b, c * BK, 0, full_b(c));
         }
-        ptx::mbar_arrive_expect_tx(full_b(s), b_bytes);
-        ptx::tma_load_2d(ptx::smem_addr(sB + s * b_bytes), &tmap_b, c * BK, nb * args.mma_n, full_b(s));
-        issued = c + 1;
-      }
-      if (!ok) {
-        for (int c = issued - ST < 0 ? 0 : issued - ST; c < issued; ++c)
-          ptx::mbar_wait_bounded(full_b(c % ST), (c / ST) & 1, status, kWaitLimitNs / 10);
+      } else {
+        long long cb = 0, issued_from = 0;
+        for (long long tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
+          const int nb = static_cast<int>(tile / args.grid_m);
+          for (int c = 0; c < nchunks; ++c, ++cb) {
+            const int s = static_cast<int>(cb % STB);
+            const long long round = cb / STB;
+            if (round > 0 && !ptx::mbar_wait_bounded(empty_b(s), static_cast<uint32_t>((round - 1) & 1), status,
+                                                      kWaitLimitNs)) {
+              ok = false;
+              break;
+            }
+            ptx::mbar_arrive_expect_tx(full_b(s), b_bytes);
+            ptx::tma_load_2d(ptx::smem_addr(sB + s * b_bytes), &tmap_b, c * BK, nb * args.mma_n, full_b(s));
+          }
+        }
+        if (!ok) {  // leave no copy in flight: wait (bounded) for the last ring's worth
+          for (long long k = (cb - STB > issued_from ? cb - STB : issued_from); k < cb; ++k)
+            ptx::mbar_wait_bounded(full_b(static_cast<int>(k % STB)), static_cast<uint32_t>((k / STB) & 1), status,
+                                   kWaitLimitNs / 10);
+        }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
+      // ---- MMA issue ----
       const uint32_t idesc = ptx::idesc_f16_f32(BM, args.mma_n);
-      for (int j = 0; j < args.nck && ok; ++j) {
-        const int hb = j % NHB;
-        if (!ptx::mbar_wait_bounded(hfull(hb), (j / NHB) & 1, status, kWaitLimitNs)) {
+      // Ring positions advance by increments (no division in this loop: the
+      // issuing thread must keep ahead of the tensor core).
+      int sb = 0, so = 0;
+      uint32_t bpar = 0, opar = 0;
+      bool b_ready = false;  // resident weights already observed
+      const uint32_t sB_addr = ptx::smem_addr(sB), sOp_addr = ptx::smem_addr(sOp);
+      const uint32_t op_stride = HALO ? halo_bytes : kATileBytes;
+      const int nops = HALO ? args.nck : nchunks;  // operand stages per tile
+      const int taps_here = HALO ? args.taps : 1;
+      long long i = 0;
+      for (long long tile = first_tile; tile < total_tiles && ok; tile += tile_step, ++i) {
+        const int a = static_cast<int>(i & 1);
+        if (i >= 2 && !ptx::mbar_wait_bounded(accempty(a), static_cast<uint32_t>(((i >> 1) - 1) & 1), status,
+                                               kWaitLimitNs)) {
           ok = false;
           break;
         }
-        int words = args.wpr - j * WC;
-        if (words > WC) words = WC;
-        const int ksteps = (words * U::L + 15) / 16;
-        const uint32_t hbase = ptx::smem_addr(sH + hb * halo_bytes);
-        for (int t = 0; t < args.taps; ++t) {
-          const int c = j * args.taps + t;
-          const int s = c % ST, round = c / ST;
-          if (!ptx::mbar_wait_bounded(full_b(s), round & 1, status, kWaitLimitNs)) {
+        ptx::tc_fence_after();  // the epilogue's reads of this accumulator are complete
+        const uint32_t tmem_d = tmem_base + static_cast<uint32_t>(a * args.mma_n);
+        uint32_t acc = 0;
+        for (int j = 0; j < nops && ok; ++j) {
+          if (!ptx::mbar_wait_bounded(opfull(so), opar, status, kWaitLimitNs)) {
             ok = false;
             break;
           }
-          ptx::tc_fence_after();
-          const int r = t / args.S, sc = t - (t / args.S) * args.S;
-          const uint64_t adesc = ptx::sw128_kmajor_desc(hbase + static_cast<uint32_t>(r * args.Wp + sc) * 128u);
-          const uint64_t bdesc = ptx::sw128_kmajor_desc(ptx::smem_addr(sB + s * b_bytes));
-          for (int kk = 0; kk < ksteps; ++kk)
-            ptx::mma_f16(tmem_base, adesc + 2 * kk, bdesc + 2 * kk, idesc, (j > 0 || t > 0 || kk > 0) ? 1u : 0u);
-          ptx::mma_commit(empty_b(s));
+          int words = (HALO ? args.wpr : args.words_total) - j * WC;
+          if (words > WC) words = WC;
+          const int ksteps = (words * U::L + 15) / 16;
+          const uint32_t opbase = sOp_addr + so * op_stride;
+          for (int t = 0; t < taps_here; ++t) {
+            uint32_t baddr;
+            if (resident) {
+              const int c = HALO ? j * args.taps + t : j;
+              if (!b_ready && !ptx::mbar_wait_bounded(full_b(c), 0, status, kWaitLimitNs)) {
+                ok = false;
+                break;
+              }
+              baddr = sB_addr + c * b_bytes;
+            } else {
+              if (!ptx::mbar_wait_bounded(full_b(sb), bpar, status, kWaitLimitNs)) {
+                ok = false;
+                break;
+              }
+              baddr = sB_addr + sb * b_bytes;
+            }
+            // No tcgen05 fence here: the operands arrived through the async
+            // proxy (TMA, or stores fenced with fence.proxy.async before the
+            // producers' arrive), which the mbarrier wait already orders.
+            const uint64_t adesc = ptx::sw128_kmajor_desc(opbase + (HALO ? s_aoff[t] : 0u));
+            const uint64_t bdesc = ptx::sw128_kmajor_desc(baddr);
+            mma_ksteps(ksteps, tmem_d, adesc, bdesc, idesc, acc);
+            acc = 1;
+            if (!resident) {
+              ptx::mma_commit(empty_b(sb));
+              if (++sb == STB) {
+                sb = 0;
+                bpar ^= 1;
+              }
+            }
+          }
+          ptx::mma_commit(opempty(so));  // the operand stage is free once these MMAs complete
+          if (++so == NO) {
+            so = 0;
+            opar ^= 1;
+          }
         }
-        ptx::mma_commit(hempty(hb));  // the halo buffer is free once these MMAs complete
+        if (ok) ptx::mma_commit(accfull(a));
+        b_ready = true;
       }
-      if (ok) ptx::mma_commit(acc_bar);
       ptx::mma_commit(drain_bar);
       int quiet = 0;
       ptx::mbar_wait_bounded(drain_bar, 0, &quiet, kWaitLimitNs);
     }
-  } else {
-    const int quad = warp & 3;
+  } else if (warp < 6) {
+    // ---- operand producers ----
     const int t = threadIdx.x - 64;  // 0..127
     const W *act = static_cast<const W *>(args.act);
-    const int wb = static_cast<int>(sizeof(W));
-    // cp.async the packed words of chunk j for this thread's halo rows
-    auto gather = [&](int j, int g) {
-      const uint32_t dst0 = ptx::smem_addr(sG + g * stage_g);
-      for (int hr = t; hr < args.HR; hr += kUnpackThreads) {
-        const long long u = v0 + hr;
-        const long long img = u / plane;
-        const long long rem = u - img * plane;
-        const int ih = static_cast<int>(rem / args.Wp) - args.pad;
-        const int iw = static_cast<int>(rem - (rem / args.Wp) * args.Wp) - args.pad;
-        const bool valid = img < args.N && ih >= 0 && ih < args.H && iw >= 0 && iw < args.W;
-        const W *px = act + ((img * args.H + ih) * args.W + iw) * args.wpr + j * WC;
-        const uint32_t dst = dst0 + hr * St::kRowBytes;
-        if (args.gather_vec) {
-          const char *src = reinterpret_cast<const char *>(valid ? px : act);
-          const uint32_t nbytes = valid ? St::kVec : 0u;
+    if constexpr (HALO) {
+      // items k = (tile i, channel chunk j), in the MMA's order
+      auto gather = [&](long long tile, int j, int slot) {
+        const uint32_t mt = static_cast<uint32_t>(tile) - fdiv(static_cast<uint32_t>(tile), args.fd_gm) * args.fd_gm.d;
+        const uint32_t v0 = mt * BM;
+        const uint32_t dst0 = ptx::smem_addr(sG + slot * stage_g);
+        for (int hr = t; hr < args.HR; hr += kUnpackThreads) {
+          const uint32_t u = v0 + hr;
+          const uint32_t img = fdiv(u, args.fd_plane);
+          const uint32_t rem = u - img * args.fd_plane.d;
+          const uint32_t ihp = fdiv(rem, args.fd_wp);
+          const int ih = static_cast<int>(ihp) - args.pad;
+          const int iw = static_cast<int>(rem - ihp * args.fd_wp.d) - args.pad;
+          const bool valid = static_cast<int>(img) < args.N && ih >= 0 && ih < args.H && iw >= 0 && iw < args.W;
+          const W *px = act + ((static_cast<long long>(img) * args.H + ih) * args.W + iw) * args.wpr + j * WC;
+          const uint32_t dst = dst0 + hr * St::kRowBytes;
+          if (args.gather_vec) {
+            const char *src = reinterpret_cast<const char *>(valid ? px : act);
+            const uint32_t nbytes = valid ? St::kVec : 0u;
 #pragma unroll
-          for (int v = 0; v < St::kBytes / St::kVec; ++v) {
-            if constexpr (St::kVec == 16)
-              ptx::cp_async_16(dst + 16 * v, src + 16 * v, nbytes);
-            else if constexpr (St::kVec == 8)
-              ptx::cp_async_8(dst + 8 * v, src + 8 * v, nbytes);
-            else
-              ptx::cp_async_4(dst + 4 * v, src + 4 * v, nbytes);
-          }
-        } else {
+            for (int v = 0; v < St::kBytes / St::kVec; ++v) {
+              if constexpr (St::kVec == 16)
+                ptx::cp_async_16(dst + 16 * v, src + 16 * v, nbytes);
+              else if constexpr (St::kVec == 8)
+                ptx::cp_async_8(dst + 8 * v, src + 8 * v, nbytes);
+              else
+                ptx::cp_async_4(dst + 4 * v, src + 4 * v, nbytes);
+            }
+          } else {
 #pragma unroll
-          for (int q = 0; q < WC; ++q) {
-            const bool in = valid && j * WC + q < args.wpr;
-            const W *src = in ? px + q : act;
-            if constexpr (sizeof(W) == 8)
-              ptx::cp_async_8(dst + 8 * q, src, in ? 8u : 0u);
-            else
-              ptx::cp_async_4(dst + 4 * q, src, in ? 4u : 0u);
+            for (int q = 0; q < WC; ++q) {
+              const bool in = valid && j * WC + q < args.wpr;
+              const W *src = in ? px + q : act;
+              if constexpr (sizeof(W) == 8)
+                ptx::cp_async_8(dst + 8 * q, src, in ? 8u : 0u);
+              else
+                ptx::cp_async_4(dst + 4 * q, src, in ? 4u : 0u);
+            }
           }
         }
-      }
-      (void)wb;
-    };
-    gather(0, 0);
-    ptx::cp_async_commit();
-    for (int j = 0; j < args.nck; ++j) {
-      if (j + 1 < args.nck) gather(j + 1, (j + 1) % NHB);
+      };
+      // the sequence of items as (tile, j) pairs
+      long long ntile = first_tile;
+      int nj = 0;
+      auto advance = [&](long long &tile, int &j) {
+        if (++j == args.nck) {
+          j = 0;
+          tile += tile_step;
+        }
+      };
+      if (ntile < total_tiles) gather(ntile, nj, 0);
       ptx::cp_async_commit();
-      ptx::cp_async_wait<1>();  // chunk j of this thread's rows has landed
-      const int hb = j % NHB;
-      if (j >= NHB) {
-        bool w_ok = true;
-        if (lane == 0) w_ok = ptx::mbar_wait_bounded(hempty(hb), ((j / NHB) - 1) & 1, status, kWaitLimitNs);
-        if (!__shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0)) {
-          ok = false;
-          break;
+      long long ctile = ntile;
+      int cj = nj;
+      advance(ntile, nj);
+      for (long long k = 0; ctile < total_tiles; ++k) {
+        if (ntile < total_tiles) gather(ntile, nj, static_cast<int>((k + 1) & 1));
+        ptx::cp_async_commit();
+        ptx::cp_async_wait<1>();  // item k of this thread's rows has landed
+        const int hb = static_cast<int>(k & 1);
+        if (k >= 2) {
+          bool w_ok = true;
+          if (lane == 0)
+            w_ok = ptx::mbar_wait_bounded(opempty(hb), static_cast<uint32_t>(((k >> 1) - 1) & 1), status, kWaitLimitNs);
+          if (!__shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0)) {
+            ok = false;
+            break;
+          }
         }
+        const uint8_t *stg = sG + (k & 1) * stage_g;
+        for (int hr = t; hr < args.HR; hr += kUnpackThreads) {
+          W cur[WC];
+          const uint8_t *src = stg + hr * St::kRowBytes;
+#pragma unroll
+          for (int v = 0; v < St::kRowBytes / 16; ++v) {
+            const uint4 q4 = *reinterpret_cast<const uint4 *>(src + 16 * v);
+            const uint32_t tw[4] = {q4.x, q4.y, q4.z, q4.w};
+#pragma unroll
+            for (int kq = 0; kq < 4; ++kq) {
+              const int byte = 16 * v + 4 * kq;
+              if (byte < St::kBytes) {
+                if constexpr (sizeof(W) == 4) {
+                  cur[byte / 4] = tw[kq];
+                } else if ((kq & 1) == 0) {
+                  cur[byte / 8] = static_cast<W>(tw[kq]) | (static_cast<W>(tw[kq + 1]) << 32);
+                }
+              }
+            }
+          }
+          U::unpack_row(cur, sOp + hb * halo_bytes, hr);
+        }
+        ptx::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(opfull(hb));
+        (void)cj;
+        ctile = ntile;
+        cj = nj;
+        advance(ntile, nj);
       }
-      const uint8_t *stg = sG + (j % NHB) * stage_g;
-      for (int hr = t; hr < args.HR; hr += kUnpackThreads) {
+      ptx::cp_async_wait<0>();
+    } else {
+      // GATHER: thread t owns row t of every A tile
+      const int row = t;
+      AGather<W, WC> g;
+      g.act = act;
+      g.H = args.H;
+      g.W_ = args.W;
+      g.wpr = args.wpr;
+      g.S = args.S;
+      g.stride = args.stride;
+      g.pad = args.pad;
+      g.words_total = args.words_total;
+      g.vec = args.gather_vec != 0;
+      auto set_tile = [&](long long tile) {
+        const uint32_t tl = static_cast<uint32_t>(tile);
+        const uint32_t mt = tl - fdiv(tl, args.fd_gm) * args.fd_gm.d;
+        const uint32_t m = mt * BM + row;
+        g.row_valid = m < static_cast<uint64_t>(args.M);
+        const uint32_t mm = g.row_valid ? m : 0u;
+        const uint32_t tq = fdiv(mm, args.fd_wo);
+        g.ow = static_cast<int>(mm - tq * args.fd_wo.d);
+        const uint32_t nq = fdiv(tq, args.fd_ho);
+        g.oh = static_cast<int>(tq - nq * args.fd_ho.d);
+        g.n = static_cast<int>(nq);
+      };
+      const uint32_t slot0 = ptx::smem_addr(sG) + row * St::kRowBytes;
+      // issue side: item (itile, ic) kGatherDepth ahead of the consume side
+      long long itile = first_tile;
+      int ic = 0;
+      if (itile < total_tiles) set_tile(itile);
+      auto issue_next = [&](int slot) {
+        if (itile < total_tiles) {
+          g.issue(ic, slot0 + slot * kSlotBytes);
+          if (++ic == nchunks) {
+            ic = 0;
+            itile += tile_step;
+            if (itile < total_tiles) set_tile(itile);
+          }
+        }
+        ptx::cp_async_commit();
+      };
+#pragma unroll 1
+      for (int d = 0; d < kGatherDepth; ++d) issue_next(d);
+      const long long items = ((total_tiles - first_tile + tile_step - 1) / tile_step) * nchunks;
+      for (long long k = 0; k < items; ++k) {
+        const int slot = static_cast<int>(k % kGatherDepth);
+        ptx::cp_async_wait<kGatherDepth - 1>();
         W cur[WC];
-        const uint8_t *src = stg + hr * St::kRowBytes;
+        const uint8_t *src = sG + slot * kSlotBytes + row * St::kRowBytes;
 #pragma unroll
         for (int v = 0; v < St::kRowBytes / 16; ++v) {
           const uint4 q4 = *reinterpret_cast<const uint4 *>(src + 16 * v);
           const uint32_t tw[4] = {q4.x, q4.y, q4.z, q4.w};
 #pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const int byte = 16 * v + 4 * k;
+          for (int kq = 0; kq < 4; ++kq) {
+            const int byte = 16 * v + 4 * kq;
             if (byte < St::kBytes) {
               if constexpr (sizeof(W) == 4) {
-                cur[byte / 4] = tw[k];
-              } else if ((k & 1) == 0) {
-                cur[byte / 8] = static_cast<W>(tw[k]) | (static_cast<W>(tw[k + 1]) << 32);
+                cur[byte / 4] = tw[kq];
+              } else if ((kq & 1) == 0) {
+                cur[byte / 8] = static_cast<W>(tw[kq]) | (static_cast<W>(tw[kq + 1]) << 32);
               }
             }
           }
         }
-        U::unpack_row(cur, sH + hb * halo_bytes, hr);
+        const int sa = static_cast<int>(k % NO);
+        const long long round = k / NO;
+        if (round > 0) {
+          bool w_ok = true;
+          if (lane == 0)
+            w_ok = ptx::mbar_wait_bounded(opempty(sa), static_cast<uint32_t>((round - 1) & 1), status, kWaitLimitNs);
+          if (!__shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0)) {
+            ok = false;
+            break;
+          }
+        }
+        U::unpack_row(cur, sOp + sa * kATileBytes, row);
+        ptx::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(opfull(sa));
+        issue_next(slot);  // refill the slot just read
       }
-      ptx::fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(hfull(hb));
+      ptx::cp_async_wait<0>();
     }
-    ptx::cp_async_wait<0>();
-    if (ok) {
+  } else {
+    // ---- epilogue ----
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    long long i = 0;
+    for (long long tile = first_tile; tile < total_tiles; tile += tile_step, ++i) {
+      const int a = static_cast<int>(i & 1);
       bool w_ok = true;
-      if (lane == 0) w_ok = ptx::mbar_wait_bounded(acc_bar, 0, status, kWaitLimitNs);
-      ok = __shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0) != 0;
-    }
-    ok = __all_sync(0xffffffffu, ok);
-    if (ok) {
+      if (lane == 0) w_ok = ptx::mbar_wait_bounded(accfull(a), static_cast<uint32_t>((i >> 1) & 1), status, kWaitLimitNs);
+      if (!__shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0)) {
+        ok = false;
+        break;
+      }
       ptx::tc_fence_after();
-      const int row = quad * 32 + lane;
-      const long long v = v0 + row;
-      const long long img = v / plane;
-      const long long rem = v - img * plane;
-      const int oh = static_cast<int>(rem / args.Wp), ow = static_cast<int>(rem - (rem / args.Wp) * args.Wp);
-      const bool valid = img < args.N && oh < args.Ho && ow < args.Wo;
-      const long long m = (img * args.Ho + oh) * args.Wo + ow;
-      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quad * 32) << 16);
-      epilogue_row(args, taddr, valid, m, nb, sH, row);
+      const uint32_t tl = static_cast<uint32_t>(tile);
+      const uint32_t nbu = fdiv(tl, args.fd_gm);
+      const int nb = static_cast<int>(nbu);
+      const uint32_t mt = tl - nbu * args.fd_gm.d;
+      bool valid;
+      long long m;
+      if (HALO) {
+        const uint32_t v = mt * BM + row;
+        const uint32_t img = fdiv(v, args.fd_plane);
+        const uint32_t rem = v - img * args.fd_plane.d;
+        const uint32_t oh = fdiv(rem, args.fd_wp);
+        const uint32_t ow = rem - oh * args.fd_wp.d;
+        valid = static_cast<int>(img) < args.N && static_cast<int>(oh) < args.Ho && static_cast<int>(ow) < args.Wo;
+        m = (static_cast<long long>(img) * args.Ho + oh) * args.Wo + ow;
+      } else {
+        m = static_cast<long long>(mt) * BM + row;
+        valid = m < args.M;
+      }
+      const uint32_t taddr = tmem_base + static_cast<uint32_t>(a * args.mma_n) + (static_cast<uint32_t>(quad * 32) << 16);
+      epilogue_row(args, taddr, valid, m, nb, sE, row);
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(accempty(a));
     }
   }
 
@@ -870,8 +960,9 @@ EncodeTiledFn encode_tiled() {
 
 struct Plan {
   int wpr, words_total, La, WC, nchunks, Kpad, NBc, n_mma, mma_n, split, nblocks, stages, Ho, Wo, gather_vec;
-  int halo, Hv, Wp, HR, nck, taps;  // halo mode (see conv_halo_kernel)
-  long long grid_m;                 // CTAs along the output positions
+  int halo, Hv, Wp, HR, nck, taps;  // halo mode (see conv_persistent_kernel)
+  long long grid_m;                 // 128-position tiles along the output
+  int stages_a, b_resident, ctas;
   long long M;
   uint32_t tmem_cols;
   size_t smem_bytes;
@@ -914,64 +1005,78 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
   p.n_mma = (p.NBc + 15) / 16 * 16;
   p.mma_n = p.split ? 2 * p.n_mma : p.n_mma;
   p.nblocks = (d->K + p.NBc - 1) / p.NBc;
-  uint32_t cols = 32;
-  while (cols < static_cast<uint32_t>(p.mma_n)) cols <<= 1;
-  p.tmem_cols = cols;
-  // packed staging ring: kGatherDepth slots of 128 rows x (chunk bytes rounded up to 16)
+  // ---- shared memory of the persistent kernel (same carve-up as the kernel)
   const int wb = fa.word_bits / 8;
   const int chunk_bytes = p.WC * wb;
-  const size_t staging = static_cast<size_t>(kGatherDepth) * BM * ((chunk_bytes + 15) / 16 * 16);
+  const int row_bytes = (chunk_bytes + 15) / 16 * 16;  // Staging::kRowBytes
   const int vec = chunk_bytes % 16 == 0 ? 16 : (chunk_bytes % 8 == 0 ? 8 : wb);
   p.gather_vec = (p.wpr % p.WC == 0) && ((static_cast<long long>(p.wpr) * wb) % vec == 0) ? 1 : 0;
-  const size_t stage_bytes = kATileBytes + static_cast<size_t>(p.mma_n) * 128;
-  const size_t fixed = 1024 + staging + 512;
-  // two CTAs per SM when at least three pipeline stages fit in half the SM's
-  // shared memory, else one CTA with a deeper ring
-  long long st = (113 * 1024 - static_cast<long long>(fixed)) / static_cast<long long>(stage_bytes);
-  if (st < 3) st = (200 * 1024 - static_cast<long long>(fixed)) / static_cast<long long>(stage_bytes);
-  if (st < 2) st = 2;
-  if (st > 6) st = 6;
-  p.stages = static_cast<int>(st);
-  p.smem_bytes = fixed + p.stages * stage_bytes;
+  const size_t bst = static_cast<size_t>(p.mma_n) * 128;
+  const bool fast_out = fo.bits != 0 && (fo.word_bits == 32 ? (32 % lanes_per_word(fo) == 0 && lanes_per_word(fo) >= 4)
+                                                            : (32 % lanes_per_word(fo) == 0 && lanes_per_word(fo) >= 8));
+  const size_t e_bytes = (fo.bits == 0 || fast_out) ? 0 : ((BM * ((p.n_mma + 31) / 32 * 32 + 4) + 15) / 16 * 16);
+  const size_t kBudget = 224 * 1024;  // below the 227 KB opt-in limit minus static shared memory
+  const size_t extra = 1024 + e_bytes + 512;  // alignment slack, epilogue rows, barriers
   p.grid_m = (p.M + BM - 1) / BM;
-
-  // Halo mode for stride-1 convolutions with several taps, when the padded
-  // virtual grid wastes little work and the halo fits in shared memory.
-  p.halo = 0;
   p.taps = d->R * d->S;
   p.nck = (p.wpr + p.WC - 1) / p.WC;
   p.Hv = d->H + 2 * d->pad;
   p.Wp = d->W + 2 * d->pad;
   p.HR = BM + (d->R - 1) * p.Wp + (d->S - 1);
-  if (d->stride == 1 && p.taps >= 2 && p.M > 0) {
-    const double virt = static_cast<double>(d->N) * p.Hv * p.Wp;
-    const double waste = virt / static_cast<double>(p.M);
-    const int nhb = p.nck > 1 ? 2 : 1;
+  p.halo = 0;
+  p.b_resident = 0;
+  p.stages_a = 0;
+  // Halo mode: stride 1, several taps, little padded-grid waste, halo fits.
+  if (d->stride == 1 && p.taps >= 2 && p.M > 0 && p.HR <= 640) {
+    const double waste = static_cast<double>(d->N) * p.Hv * p.Wp / static_cast<double>(p.M);
     const size_t halo_bytes = static_cast<size_t>((p.HR + 7) / 8 * 8) * 128;
-    const size_t stage_g = static_cast<size_t>((p.HR * ((chunk_bytes + 15) / 16 * 16) + 15) / 16 * 16);
-    const size_t bst = static_cast<size_t>(p.mma_n) * 128;
-    const size_t hfixed = 1024 + nhb * (halo_bytes + stage_g) + 512;
+    const size_t stage_g = static_cast<size_t>((p.HR * row_bytes + 15) / 16 * 16);
+    const size_t fixed = extra + 2 * halo_bytes + 2 * stage_g;
     const int ntiles_b = p.nck * p.taps;
-    long long hst = (113 * 1024 - static_cast<long long>(hfixed)) / static_cast<long long>(bst);
-    if (hst < 4) hst = (200 * 1024 - static_cast<long long>(hfixed)) / static_cast<long long>(bst);
-    if (hst > ntiles_b) hst = ntiles_b;
-    if (hst > 16) hst = 16;
-    if (waste <= 1.16 && p.HR <= 640 && hst >= 2) {
+    if (waste <= 1.16 && fixed + 2 * bst <= kBudget) {
       p.halo = 1;
-      p.stages = static_cast<int>(hst);
-      p.smem_bytes = hfixed + p.stages * bst;
       p.nchunks = ntiles_b;
       p.Kpad = ntiles_b * BK;
       p.grid_m = (static_cast<long long>(d->N) * p.Hv * p.Wp + BM - 1) / BM;
-      p.gather_vec = (p.wpr % p.WC == 0) && ((static_cast<long long>(p.wpr) * wb) % vec == 0) ? 1 : 0;
+      if (p.nblocks == 1 && fixed + ntiles_b * bst <= kBudget) {
+        p.b_resident = 1;
+        p.stages = ntiles_b;
+      } else {
+        long long st = static_cast<long long>((kBudget - fixed) / bst);
+        p.stages = static_cast<int>(st > 8 ? 8 : st);
+      }
+      p.smem_bytes = fixed + p.stages * bst;
     }
   }
+  if (!p.halo) {
+    const size_t staging = static_cast<size_t>(kGatherDepth) * BM * row_bytes;
+    for (int sta = 4; sta >= 2; --sta) {
+      const size_t fixed = extra + sta * static_cast<size_t>(kATileBytes) + staging;
+      if (fixed + 2 * bst > kBudget) continue;
+      p.stages_a = sta;
+      if (p.nblocks == 1 && fixed + p.nchunks * bst <= kBudget) {
+        p.b_resident = 1;
+        p.stages = p.nchunks;
+      } else {
+        long long st = static_cast<long long>((kBudget - fixed) / bst);
+        p.stages = static_cast<int>(st > 8 ? 8 : st);
+      }
+      p.smem_bytes = fixed + p.stages * bst;
+      break;
+    }
+    if (p.stages_a == 0) return SAMD_EUNSUP;  // operand tiles do not fit (not reached for N <= 256)
+  }
+  uint32_t cols = 32;
+  while (cols < static_cast<uint32_t>(2 * p.mma_n)) cols <<= 1;  // two accumulators
+  p.tmem_cols = cols;
   p.ws_bytes = static_cast<size_t>(p.nblocks) * p.mma_n * p.Kpad * sizeof(__half);
   return SAMD_OK;
 }
 
 // cudaFuncSetAttribute once per (kernel, device), so that launches made
 // while a stream is being captured into a graph issue no other CUDA call.
+// The dynamic limit is the per-block maximum minus the kernel's static
+// shared memory. Returns cudaErrorInvalidValue if `smem` does not fit.
 cudaError_t ensure_smem_attr(const void *kern, size_t smem) {
   static std::mutex mu;
   static const void *done_fn[256];
@@ -983,30 +1088,32 @@ cudaError_t ensure_smem_attr(const void *kern, size_t smem) {
   if (e != cudaSuccess) return e;
   std::lock_guard<std::mutex> lock(mu);
   for (int i = 0; i < n_done; ++i)
-    if (done_fn[i] == kern && done_dev[i] == dev && done_smem[i] >= smem) return cudaSuccess;
-  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+    if (done_fn[i] == kern && done_dev[i] == dev) return smem <= done_smem[i] ? cudaSuccess : cudaErrorInvalidValue;
+  int optin = 0;
+  e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
   if (e != cudaSuccess) return e;
-  for (int i = 0; i < n_done; ++i)
-    if (done_fn[i] == kern && done_dev[i] == dev) {
-      done_smem[i] = 200 * 1024;
-      return cudaSuccess;
-    }
+  cudaFuncAttributes fa;
+  e = cudaFuncGetAttributes(&fa, kern);
+  if (e != cudaSuccess) return e;
+  const size_t limit = static_cast<size_t>(optin) - fa.sharedSizeBytes;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(limit));
+  if (e != cudaSuccess) return e;
   if (n_done < 256) {
     done_fn[n_done] = kern;
     done_dev[n_done] = dev;
-    done_smem[n_done] = 200 * 1024;
+    done_smem[n_done] = limit;
     ++n_done;
   }
-  return cudaSuccess;
+  return smem <= limit ? cudaSuccess : cudaErrorInvalidValue;
 }
 
 template <typename W, int BITS, bool SIGNED>
 cudaError_t launch_conv_variant(const CUtensorMap &tmap, const ConvArgs &args, dim3 grid, size_t smem,
                                 cudaStream_t s) {
-  auto kern = args.HR > 0 ? conv_halo_kernel<W, BITS, SIGNED> : conv_tc_kernel<W, BITS, SIGNED>;
+  auto kern = args.HR > 0 ? conv_persistent_kernel<W, BITS, SIGNED, true> : conv_persistent_kernel<W, BITS, SIGNED, false>;
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void *>(kern), smem);
   if (e != cudaSuccess) return e;
-  kern<<<grid, kThreads, smem, s>>>(tmap, args);
+  kern<<<grid, kPThreads, smem, s>>>(tmap, args);
   return cudaGetLastError();
 }
 
@@ -1138,6 +1245,10 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   a.mma_n = p.mma_n;
   a.split = p.split;
   a.stages = p.stages;
+  a.stages_a = p.stages_a;
+  a.b_resident = p.b_resident;
+  a.grid_m = p.grid_m;
+  a.nblocks = p.nblocks;
   a.gather_vec = p.gather_vec;
   a.tmem_cols = p.tmem_cols;
   a.out_bits = packed_out ? fo.bits : 8;
@@ -1158,7 +1269,19 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   a.HR = p.halo ? p.HR : 0;  // 0 selects the gather kernel
   a.nck = p.nck;
   a.taps = p.taps;
-  dim3 grid(static_cast<unsigned>(p.grid_m), static_cast<unsigned>(p.nblocks));
+  // the kernel's index math runs in 32 bits
+  if (static_cast<long long>(d->N) * p.Hv * p.Wp + p.HR + BM >= (1LL << 31) || p.M >= (1LL << 31) ||
+      p.grid_m * p.nblocks >= (1LL << 31))
+    return SAMD_EUNSUP;
+  a.fd_plane = make_fastdiv(static_cast<uint32_t>(p.Hv * p.Wp));
+  a.fd_wp = make_fastdiv(static_cast<uint32_t>(p.Wp));
+  a.fd_wo = make_fastdiv(static_cast<uint32_t>(p.Wo));
+  a.fd_ho = make_fastdiv(static_cast<uint32_t>(p.Ho));
+  a.fd_gm = make_fastdiv(static_cast<uint32_t>(p.grid_m));
+  const long long total_tiles = p.grid_m * p.nblocks;
+  long long ctas = sm_count();
+  if (ctas > total_tiles) ctas = total_tiles;
+  dim3 grid(static_cast<unsigned>(ctas));
   cudaError_t e = fa.word_bits == 32 ? launch_conv_word<uint32_t>(fa, tmap, a, grid, p.smem_bytes, s)
                                      : launch_conv_word<uint64_t>(fa, tmap, a, grid, p.smem_bytes, s);
   return e == cudaSuccess ? SAMD_OK : SAMD_ECUDA;
