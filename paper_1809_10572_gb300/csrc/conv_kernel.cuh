@@ -1,0 +1,996 @@
+// conv_kernel.cuh -- the persistent tcgen05 convolution kernel (device code
+// shared by the translation units that instantiate it).
+//
+// The paper's DNN convolution (section 7, Fig. 12, direct-sum2d) is
+//   acc[n][k][ho][wo] = sum_{c,r,s} act[n][c][ho*st-p+r][wo*st-p+s] * wt[k][c][r][s].
+// Here it is the GEMM D[M x K] = A[M x Kg] * B[K x Kg]^T with M = N*Ho*Wo
+// output pixels and a reduction index Kg running over (tap, packed word,
+// lane). Activations and weights stay packed in HBM and L2 and are widened
+// only in shared memory, right before the MMA (the "unpack to the native
+// type" baseline of section 7, moved on-chip).
+//
+// Exactness. sm_103a has no integer MMA, so lanes are widened to a float
+// type whose every value in play is an exact integer, and the fp32
+// accumulators hold exact integers while every partial sum stays below 2^24:
+//   e4m3 (kind::f8f6f4, K = 32 per MMA) when |a| <= 16 and |w| <= 16 (lane
+//        widths up to 4 bits, and signed 5-bit lanes); half the shared-memory
+//        bytes of fp16 per product, twice the tensor rate;
+//   fp16 (kind::f16, K = 16 per MMA) otherwise: every integer of [-128, 255].
+// When R*S*C*max|a|*max|w| reaches 2^24 (wide weights over many taps), the
+// fp16 weights are split into two 4-bit digits w = 16*hi + lo stacked along
+// the MMA's N; the epilogue forms 16*hi + lo in int32.
+//
+// Both operand types use rows of 64 reduction positions: 128-byte rows with
+// the 128-byte swizzle (fp16) or 64-byte rows with the 64-byte swizzle
+// (e4m3). An MMA consumes 32 bytes of a row either way, so the descriptors
+// advance by the same 32 bytes per MMA.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_fp16.h>
+
+#include <cstring>
+#include <utility>
+
+#include "samd_internal.cuh"
+#include "tc_ptx.cuh"
+
+namespace samd {
+namespace conv {
+
+constexpr int BM = 128;  // output pixels per tile = MMA M = TMEM lanes
+constexpr int BK = 64;   // reduction positions per chunk = one operand row
+constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s
+constexpr int kGatherDepth = 4;                    // packed chunks in flight per producer thread
+constexpr int kProdWarps = 8;                      // operand producers
+constexpr int kEpiWarps = 8;                       // epilogue
+constexpr int kProdThreads = 32 * kProdWarps;
+constexpr int kThreads = 32 * (2 + kProdWarps + kEpiWarps);
+constexpr int kFirstEpiWarp = 2 + kProdWarps;
+
+template <bool FP8>
+struct OpTraits {
+  static constexpr int kRowBytes = FP8 ? 64 : 128;  // one row of BK positions
+  static constexpr int kKPerMma = FP8 ? 32 : 16;
+  static constexpr uint32_t kTileBytes = BM * kRowBytes;
+  // 16-byte chunk c of row r (rows kRowBytes apart from a 1024-byte-aligned base)
+  __device__ static __forceinline__ int swz(int r, int c) { return FP8 ? (c ^ ((r >> 1) & 3)) : (c ^ (r & 7)); }
+  __device__ static __forceinline__ uint64_t desc(uint32_t saddr) {
+    return FP8 ? ptx::sw64_kmajor_desc(saddr) : ptx::sw128_kmajor_desc(saddr);
+  }
+};
+
+__host__ __device__ constexpr bool pair16(int bits) { return bits == 1 || bits == 2 || bits == 4 || bits == 8; }
+
+// The lane of a packed word held by reduction position `pos` (0 <= pos < L)
+// of that word. For lane widths dividing 16, positions 2p and 2p+1 hold
+// lanes p and p + 16/bits of the same 32-bit half, which sit exactly 16 bits
+// apart, so one masked shift widens both at once. Other widths keep lane
+// order. A and B use the same map, so the dot products are unchanged.
+__host__ __device__ constexpr int kpos_lane(int bits, int pos) {
+  if (pair16(bits)) {
+    int g = 32 / bits, half = pos / g, jj = pos % g;
+    return half * g + jj / 2 + (jj & 1) * (g / 2);
+  }
+  return pos;
+}
+
+// n / d for 0 <= n < 2^31 by one multiply-high, an add and a shift:
+// l = ceil(log2 d), m = floor(2^32 (2^l - d) / d) + 1, q = (umulhi(m, n) + n) >> l.
+struct FastDiv {
+  uint32_t m;
+  int l;
+  uint32_t d;
+};
+
+inline FastDiv make_fastdiv(uint32_t d) {
+  int l = 0;
+  while ((uint64_t(1) << l) < d) ++l;
+  const uint64_t m = ((uint64_t(1) << 32) * ((uint64_t(1) << l) - d)) / d + 1;
+  return FastDiv{static_cast<uint32_t>(m), l, d};
+}
+
+__device__ __forceinline__ uint32_t fdiv(uint32_t n, const FastDiv &f) { return (__umulhi(f.m, n) + n) >> f.l; }
+
+struct ConvArgs {
+  const void *act;
+  int32_t *acc_out;
+  void *packed_out;
+  int *status;  // sticky SAMD_ETIMEOUT record of this device
+  int N, C, H, W, K, R, S, stride, pad, Ho, Wo;
+  long long M;
+  int wpr;          // activation words per pixel
+  int words_total;  // R * S * wpr: reduction length in packed words (GATHER)
+  int nchunks;      // weight tiles per output tile
+  int NBc;          // output channels per channel block
+  int n_mma;        // NBc rounded up to 16
+  int mma_n;        // MMA N: n_mma, or 2 * n_mma with split weight digits
+  int split;        // 1: accumulator columns [0, n_mma) hold hi digits, [n_mma, 2 n_mma) lo digits
+  int stages;       // weight tiles in flight (or resident)
+  int stages_a;     // GATHER: A tiles in flight
+  int b_resident;   // 1: all weight tiles of the layer stay in shared memory
+  long long grid_m; // 128-position tiles along the output
+  int nblocks;      // channel blocks
+  int gather_vec;   // AGather::vec
+  uint32_t tmem_cols;
+  int out_bits, out_signed, out_lane_w, out_L, out_word64, out_wpr;
+  int out_fast;     // output lanes per word when they divide 32 (packing in registers), else 0
+  int shift;
+  // HALO (stride 1): virtual output grid of N x Hv x Wp positions. A tile of
+  // 128 consecutive positions v0.. reads nseg segments of the input grid:
+  // segment g holds seg_used rows starting at virtual row v0 + g * Wp and
+  // occupies seg_rows rows of the halo buffer; tap (r, s) reads the 128 rows
+  // starting at halo row r * row_step + s.
+  int Hv, Wp;
+  int nseg, seg_rows, seg_used, row_step;
+  int nck;   // channel chunks per pixel (ceil(wpr / WC))
+  int taps;  // R * S
+  FastDiv fd_plane, fd_wp;  // / (Hv * Wp), / Wp
+  FastDiv fd_seg;           // / seg_rows
+  FastDiv fd_wo, fd_ho;     // output pixel index -> (n, oh, ow)
+  FastDiv fd_gm;            // tile -> (channel block, position tile)
+  // shared memory carve-up (bytes from the 1024-byte-aligned base)
+  uint32_t op_stride;  // one halo buffer or one A tile
+  uint32_t off_b, b_bytes, off_g, g_stride, off_e, off_bar;
+};
+
+__device__ __forceinline__ uint32_t hsub2_bits(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+
+// two fp16 integers (|v| <= 16, exact in e4m3) -> two e4m3 bytes, low half first
+__device__ __forceinline__ uint32_t f16x2_to_e4m3x2(uint32_t h) {
+  uint16_t r;
+  asm("cvt.rn.satfinite.e4m3x2.f16x2 %0, %1;" : "=h"(r) : "r"(h));
+  return r;
+}
+
+// Widening of one 64-position row of the A operand (one pixel, one chunk).
+template <typename W, int BITS, bool SIGNED, bool FP8>
+struct AUnpack {
+  static constexpr int WB = WordTraits<W>::kBits;
+  static constexpr int L = WB / BITS;
+  static constexpr int WC = BK / L;        // packed words per chunk
+  static constexpr int KUSED = WC * L;     // positions holding lanes; the rest are zero
+  static constexpr uint32_t LM = (1u << BITS) - 1;
+  static constexpr uint32_t OFF = SIGNED ? (1u << (BITS - 1)) : 0u;  // offset-binary zero
+  static constexpr uint32_t BIAS = 0x6400u + OFF;                   // fp16 bits of 1024 + OFF
+  static constexpr uint32_t BIAS2 = BIAS | (BIAS << 16);
+
+  static constexpr W sign_mask() {
+    W m = 0;
+    for (int i = 0; i < L; ++i) m |= W(1) << (i * BITS + BITS - 1);
+    return m;
+  }
+
+  template <int POS>
+  __device__ static __forceinline__ uint32_t field(W w) {
+    return static_cast<uint32_t>(w >> (kpos_lane(BITS, POS) * BITS)) & LM;
+  }
+
+  // A lane pattern v (offset binary when signed) becomes fp16 1024 + v by
+  // or-ing it into the mantissa of 1024.0; subtracting 1024 + OFF leaves the
+  // lane's value exactly. A zero word (padding) therefore widens to zeros.
+  template <int P>
+  __device__ static __forceinline__ uint32_t pair(const W (&w)[WC]) {
+    constexpr int j0 = 2 * P, j1 = 2 * P + 1;
+    if constexpr (j0 >= KUSED) {
+      return 0u;
+    } else if constexpr (pair16(BITS)) {
+      constexpr int q = j0 / L, pos = j0 % L, g = 32 / BITS, half = pos / g;
+      constexpr int lane0 = kpos_lane(BITS, pos) - half * g;
+      const uint32_t x = static_cast<uint32_t>(w[q] >> (half * 32));
+      const uint32_t t = ((x >> (lane0 * BITS)) & (LM | (LM << 16))) | 0x64006400u;
+      return hsub2_bits(t, BIAS2);
+    } else {
+      const uint32_t v0 = field<j0 % L>(w[j0 / L]);
+      uint32_t v1 = OFF;
+      if constexpr (j1 < KUSED) v1 = field<j1 % L>(w[j1 / L]);
+      return hsub2_bits(v0 | (v1 << 16) | 0x64006400u, BIAS2);
+    }
+  }
+
+  template <int... P>
+  __device__ static __forceinline__ void pairs(const W (&w)[WC], uint32_t (&h)[32],
+                                               std::integer_sequence<int, P...>) {
+    ((h[P] = pair<P>(w)), ...);
+  }
+
+  // Widen one pixel's chunk and store it as row `row` of a swizzled K-major
+  // operand whose rows are OpTraits::kRowBytes apart.
+  __device__ static __forceinline__ void unpack_row(W (&w)[WC], uint8_t *tile, int row) {
+    using T = OpTraits<FP8>;
+    if constexpr (SIGNED) {
+#pragma unroll
+      for (int q = 0; q < WC; ++q) w[q] ^= sign_mask();
+    }
+    uint32_t h[32];
+    pairs(w, h, std::make_integer_sequence<int, 32>{});
+    uint8_t *rp = tile + row * T::kRowBytes;
+    if constexpr (FP8) {
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint32_t b[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          b[k] = f16x2_to_e4m3x2(h[8 * c + 2 * k]) | (f16x2_to_e4m3x2(h[8 * c + 2 * k + 1]) << 16);
+        *reinterpret_cast<uint4 *>(rp + (T::swz(row, c) << 4)) = make_uint4(b[0], b[1], b[2], b[3]);
+      }
+    } else {
+#pragma unroll
+      for (int c = 0; c < 8; ++c)
+        *reinterpret_cast<uint4 *>(rp + (T::swz(row, c) << 4)) =
+            make_uint4(h[4 * c], h[4 * c + 1], h[4 * c + 2], h[4 * c + 3]);
+    }
+  }
+};
+
+// Bytes of one pixel-chunk row in the packed staging buffers (a multiple of 16).
+template <typename W, int WC>
+struct Staging {
+  static constexpr int kBytes = WC * static_cast<int>(sizeof(W));
+  static constexpr int kRowBytes = (kBytes + 15) / 16 * 16;
+  // widest cp.async that divides a whole chunk held by one pixel
+  static constexpr int kVec = kBytes % 16 == 0 ? 16 : (kBytes % 8 == 0 ? 8 : static_cast<int>(sizeof(W)));
+};
+
+// Copies a pixel-chunk of kBytes from `src` (vector-aligned) to staging with
+// cp.async; nbytes = 0 zero-fills it.
+template <typename W, int WC>
+__device__ __forceinline__ void stage_chunk(uint32_t dst, const char *src, uint32_t valid) {
+  using St = Staging<W, WC>;
+#pragma unroll
+  for (int v = 0; v < St::kBytes / St::kVec; ++v) {
+    if constexpr (St::kVec == 16)
+      ptx::cp_async_16(dst + 16 * v, src + 16 * v, valid ? 16u : 0u);
+    else if constexpr (St::kVec == 8)
+      ptx::cp_async_8(dst + 8 * v, src + 8 * v, valid ? 8u : 0u);
+    else
+      ptx::cp_async_4(dst + 4 * v, src + 4 * v, valid ? 4u : 0u);
+  }
+}
+
+// Reads a staged pixel-chunk back into words.
+template <typename W, int WC>
+__device__ __forceinline__ void load_staged(const uint8_t *src, W (&cur)[WC]) {
+  using St = Staging<W, WC>;
+#pragma unroll
+  for (int v = 0; v < St::kRowBytes / 16; ++v) {
+    const uint4 q4 = *reinterpret_cast<const uint4 *>(src + 16 * v);
+    const uint32_t tw[4] = {q4.x, q4.y, q4.z, q4.w};
+#pragma unroll
+    for (int kq = 0; kq < 4; ++kq) {
+      const int byte = 16 * v + 4 * kq;
+      if (byte < St::kBytes) {
+        if constexpr (sizeof(W) == 4) {
+          cur[byte / 4] = tw[kq];
+        } else if ((kq & 1) == 0) {
+          cur[byte / 8] = static_cast<W>(tw[kq]) | (static_cast<W>(tw[kq + 1]) << 32);
+        }
+      }
+    }
+  }
+}
+
+// Gathers the packed words of one pixel's chunk into shared memory with
+// cp.async: word kw of the reduction is word (kw mod wpr) of the input pixel
+// at tap kw / wpr; taps outside the image and words past the end are
+// zero-filled (source size 0).
+template <typename W, int WC>
+struct AGather {
+  const W *act;
+  int H, W_, wpr, S, stride, pad, words_total;
+  int n, oh, ow;
+  bool row_valid;
+  bool vec;  // every chunk lies inside one pixel at a kVec-aligned offset
+
+  __device__ __forceinline__ const W *pixel(int tap, bool &valid) const {
+    int r = tap / S, s = tap - (tap / S) * S;
+    int ih = oh * stride - pad + r, iw = ow * stride - pad + s;
+    valid = row_valid && ih >= 0 && ih < H && iw >= 0 && iw < W_;
+    return act + ((static_cast<long long>(n) * H + ih) * W_ + iw) * wpr;
+  }
+
+  __device__ __forceinline__ void issue(int chunk, uint32_t dst) const {
+    const int kw0 = chunk * WC;
+    int tap = kw0 / wpr, wi = kw0 - tap * wpr;
+    bool valid;
+    const W *px = pixel(tap, valid);
+    if (vec) {
+      stage_chunk<W, WC>(dst, reinterpret_cast<const char *>(valid ? px + wi : act), valid ? 1u : 0u);
+      return;
+    }
+#pragma unroll
+    for (int q = 0; q < WC; ++q) {
+      const bool in = valid && kw0 + q < words_total;
+      const W *src = in ? px + wi : act;
+      if constexpr (sizeof(W) == 8)
+        ptx::cp_async_8(dst + 8 * q, src, in ? 8u : 0u);
+      else
+        ptx::cp_async_4(dst + 4 * q, src, in ? 4u : 0u);
+      if (++wi == wpr) {
+        wi = 0;
+        ++tap;
+        px = pixel(tap, valid);
+      }
+    }
+  }
+};
+
+// Packs 32 requantized lane patterns (zero past `cnt`) into 32 / LO words of
+// LO lanes each and stores them; LO divides 32, so every word of the
+// 32-channel group is whole.
+template <int LO, typename WO>
+__device__ __forceinline__ void pack_regs(const uint32_t (&y)[32], int lane_w, int cnt, WO *dst) {
+  constexpr int NW = 32 / LO;  // words of this 32-channel group
+  WO w[NW];
+#pragma unroll
+  for (int k = 0; k < NW; ++k) {
+    w[k] = 0;
+#pragma unroll
+    for (int l = 0; l < LO; ++l) w[k] |= static_cast<WO>(y[k * LO + l]) << (l * lane_w);
+  }
+  constexpr int kWordBytes = static_cast<int>(sizeof(WO));
+  if (cnt == 32 && (NW * kWordBytes) % 16 == 0 && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+#pragma unroll
+    for (int v = 0; v < NW * kWordBytes / 16; ++v) {
+      uint4 q;
+      memcpy(&q, reinterpret_cast<const uint8_t *>(w) + 16 * v, 16);
+      reinterpret_cast<uint4 *>(dst)[v] = q;
+    }
+  } else {
+#pragma unroll
+    for (int k = 0; k < NW; ++k)
+      if (k * LO < cnt) dst[k] = w[k];
+  }
+}
+
+// Epilogue of one accumulator row (one output pixel m) of channel block nb,
+// for the 32-column groups g = half, half + 2, ...: fp32 accumulators ->
+// exact int32 -> optional int32 store, optional requantize-and-pack. Called
+// by whole warps (tcgen05.ld is collective). Output formats whose words do
+// not divide a 32-channel group go through one byte per channel in `ebuf`
+// (128 rows x ebytes): half 1 writes its bytes and arrives on `ebar_full`,
+// half 0 waits for it, assembles the row's words and arrives on `ebar_free`,
+// which half 1 awaits before it writes the next tile's bytes (tile index i).
+// Returns false when a bounded wait gave up.
+__device__ __forceinline__ bool epilogue_row(const ConvArgs &args, uint32_t taddr, bool row_valid, long long m,
+                                             int nb, uint8_t *ebuf, int row, int half, uint32_t ebar_full,
+                                             uint32_t ebar_free, long long i) {
+  const int lane = threadIdx.x & 31;
+  const int ch0 = nb * args.NBc;
+  const int nvalid = args.K - ch0 < args.NBc ? args.K - ch0 : args.NBc;
+  const bool vec_ok = (args.K % 4 == 0) && (ch0 % 4 == 0);
+  const int lo = lane_lo(args.out_bits, args.out_signed), hi = lane_hi(args.out_bits, args.out_signed);
+  const uint32_t omask = (1u << args.out_bits) - 1;
+  const bool bytes_path = args.packed_out && !args.out_fast;
+  volatile int *status = args.status;
+  auto wait_lane0 = [&](uint32_t bar, uint32_t parity) {
+    bool w_ok = true;
+    if (lane == 0) w_ok = ptx::mbar_wait_bounded(bar, parity, status, kWaitLimitNs);
+    return __shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0) != 0;
+  };
+  if (bytes_path && half == 1 && i >= 1 && !wait_lane0(ebar_free, static_cast<uint32_t>((i - 1) & 1))) return false;
+  // A row holds whole 32-channel groups plus 4 bytes: an odd number of 32-bit
+  // words, so the warp's 4-byte stores fall in distinct banks.
+  const int ebytes = (args.n_mma + 31) / 32 * 32 + 4;
+  uint8_t *erow = ebuf + row * ebytes;
+  for (int col = 32 * half; col < nvalid; col += 64) {
+    uint32_t r[32];
+    int v[32];
+    ptx::tmem_ld_32x32b_x32(taddr + col, r);
+    if (args.split) {  // acc = 16 * hi + lo
+      uint32_t r2[32];
+      ptx::tmem_ld_32x32b_x32(taddr + args.n_mma + col, r2);
+      ptx::tmem_wait_ld();
+#pragma unroll
+      for (int k = 0; k < 32; ++k)
+        v[k] = 16 * __float2int_rn(__uint_as_float(r[k])) + __float2int_rn(__uint_as_float(r2[k]));
+    } else {
+      ptx::tmem_wait_ld();
+#pragma unroll
+      for (int k = 0; k < 32; ++k) v[k] = __float2int_rn(__uint_as_float(r[k]));
+    }
+    if (!row_valid) continue;
+    const int cnt = nvalid - col < 32 ? nvalid - col : 32;
+    if (args.acc_out) {
+      int32_t *dst = args.acc_out + m * args.K + ch0 + col;
+      if (cnt == 32 && vec_ok) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          reinterpret_cast<int4 *>(dst)[k] = make_int4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+      } else {
+#pragma unroll
+        for (int k = 0; k < 32; ++k)
+          if (k < cnt) dst[k] = v[k];
+      }
+    }
+    if (args.packed_out) {
+      uint32_t y[32];
+#pragma unroll
+      for (int k = 0; k < 32; ++k)
+        y[k] = k < cnt ? static_cast<uint32_t>(clamp_int(v[k] >> args.shift, lo, hi)) & omask : 0u;
+      if (args.out_fast) {
+        const long long w0 = m * args.out_wpr + (ch0 + col) / args.out_L;
+        const int lw = args.out_lane_w;
+        if (args.out_word64) {
+          uint64_t *dst = static_cast<uint64_t *>(args.packed_out) + w0;
+          switch (args.out_fast) {
+            case 8: pack_regs<8>(y, lw, cnt, dst); break;
+            case 16: pack_regs<16>(y, lw, cnt, dst); break;
+            default: pack_regs<32>(y, lw, cnt, dst); break;
+          }
+        } else {
+          uint32_t *dst = static_cast<uint32_t *>(args.packed_out) + w0;
+          switch (args.out_fast) {
+            case 4: pack_regs<4>(y, lw, cnt, dst); break;
+            case 8: pack_regs<8>(y, lw, cnt, dst); break;
+            case 16: pack_regs<16>(y, lw, cnt, dst); break;
+            default: pack_regs<32>(y, lw, cnt, dst); break;
+          }
+        }
+      } else {
+#pragma unroll
+        for (int k4 = 0; k4 < 8; ++k4)
+          *reinterpret_cast<uint32_t *>(erow + col + 4 * k4) =
+              y[4 * k4] | (y[4 * k4 + 1] << 8) | (y[4 * k4 + 2] << 16) | (y[4 * k4 + 3] << 24);
+      }
+    }
+  }
+  if (!bytes_path) return true;
+  if (half == 1) {
+    __syncwarp();
+    if (lane == 0) ptx::mbar_arrive(ebar_full);  // this tile's bytes of the other half are written
+    return true;
+  }
+  if (!wait_lane0(ebar_full, static_cast<uint32_t>(i & 1))) return false;
+  // each output word packs L consecutive channels of this row
+  if (row_valid) {
+    const int Lo = args.out_L, lw = args.out_lane_w;
+    const int nwords = (nvalid + Lo - 1) / Lo;
+    const long long w0 = m * args.out_wpr + ch0 / Lo;
+    if (args.out_word64) {
+      uint64_t *dst = static_cast<uint64_t *>(args.packed_out) + w0;
+      for (int j = 0; j < nwords; ++j) {
+        const int c0 = j * Lo, cn = nvalid - c0 < Lo ? nvalid - c0 : Lo;
+        uint64_t wv = 0;
+        for (int l = 0; l < cn; ++l) wv |= static_cast<uint64_t>(erow[c0 + l]) << (l * lw);
+        dst[j] = wv;
+      }
+    } else {
+      uint32_t *dst = static_cast<uint32_t *>(args.packed_out) + w0;
+      for (int j = 0; j < nwords; ++j) {
+        const int c0 = j * Lo, cn = nvalid - c0 < Lo ? nvalid - c0 : Lo;
+        uint32_t wv = 0;
+        for (int l = 0; l < cn; ++l) wv |= static_cast<uint32_t>(erow[c0 + l]) << (l * lw);
+        dst[j] = wv;
+      }
+    }
+  }
+  __syncwarp();
+  if (lane == 0) ptx::mbar_arrive(ebar_free);  // the bytes may be overwritten
+  return true;
+}
+
+// Issues `ksteps` (1..4) MMAs of one operand row as straight-line code.
+template <bool FP8>
+__device__ __forceinline__ void mma_op(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  if constexpr (FP8)
+    ptx::mma_f8(d, a, b, idesc, acc);
+  else
+    ptx::mma_f16(d, a, b, idesc, acc);
+}
+
+template <bool FP8>
+__device__ __forceinline__ void mma_ksteps(int ksteps, uint32_t d, uint64_t a, uint64_t b, uint32_t idesc,
+                                           uint32_t acc) {
+  switch (ksteps) {
+    case 4:
+      mma_op<FP8>(d, a, b, idesc, acc);
+      mma_op<FP8>(d, a + 2, b + 2, idesc, 1u);
+      mma_op<FP8>(d, a + 4, b + 4, idesc, 1u);
+      mma_op<FP8>(d, a + 6, b + 6, idesc, 1u);
+      break;
+    case 3:
+      mma_op<FP8>(d, a, b, idesc, acc);
+      mma_op<FP8>(d, a + 2, b + 2, idesc, 1u);
+      mma_op<FP8>(d, a + 4, b + 4, idesc, 1u);
+      break;
+    case 2:
+      mma_op<FP8>(d, a, b, idesc, acc);
+      mma_op<FP8>(d, a + 2, b + 2, idesc, 1u);
+      break;
+    default:
+      mma_op<FP8>(d, a, b, idesc, acc);
+      break;
+  }
+}
+
+// Issues the MMAs of all `taps` taps of one operand stage with resident
+// weights: tap t reads weight tile t (b advances by b_step16) and the A
+// operand one row further on, skipping a_skip16 at the end of each filter
+// row (HALO); straight-line issue keeps the tensor core fed. Descriptors
+// advance in 16-byte units of their start-address field.
+template <bool FP8>
+__device__ __forceinline__ void issue_taps(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, int ksteps, int taps,
+                                           int S, uint32_t a_row16, uint32_t a_skip16, uint32_t b_step16,
+                                           uint32_t acc) {
+  int s = 0;
+  for (int t = 0; t < taps; ++t) {
+    mma_ksteps<FP8>(ksteps, d, a, b, idesc, acc);
+    acc = 1;
+    b += b_step16;
+    a += a_row16;
+    if (++s == S) {
+      s = 0;
+      a += a_skip16;
+    }
+  }
+}
+
+// ---- the persistent convolution kernel ----------------------------------------
+//
+// One CTA per SM loops over output tiles (tile = blockIdx.x + i * gridDim.x;
+// tile = nb * grid_m + mt: channel block nb, 128-position tile mt). Eighteen
+// warps with fixed roles, connected by mbarrier rings:
+//   warp 0      TMEM allocation; lane 0 streams weight tiles with TMA. When
+//               the layer has one channel block and all its weight tiles fit,
+//               they are loaded once and stay resident.
+//   warp 1      issues tcgen05.mma (one elected lane) into one of two TMEM
+//               accumulators, so tile i+1 accumulates while the epilogue
+//               drains tile i.
+//   warps 2-9   operand producers.
+//               HALO: for each (tile, channel chunk) the halo rows the tile
+//               needs are gathered with cp.async and widened once into one of
+//               two halo buffers; every tap reads the halo through a
+//               descriptor shifted by r * row_step + s rows.
+//               GATHER: two groups of four warps take alternate (tile, chunk)
+//               items; each thread gathers its pixel's packed words (implicit
+//               im2col, zero padding) through a cp.async ring and widens them
+//               into a ring of A tiles.
+//   warps 10-17 epilogue: tcgen05.ld, exact int32, optional int32 store,
+//               optional requantize-and-pack; warp w reads TMEM lanes of
+//               quadrant w % 4, the two warps of a quadrant take alternate
+//               32-column groups.
+// Every wait is bounded; a role that gives up records SAMD_ETIMEOUT and stops.
+template <typename W, int BITS, bool SIGNED, bool HALO, bool FP8>
+__global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant__ CUtensorMap tmap_b,
+                                                           const ConvArgs args) {
+  using U = AUnpack<W, BITS, SIGNED, FP8>;
+  using T = OpTraits<FP8>;
+  constexpr int WC = U::WC;
+  using St = Staging<W, WC>;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ int s_skip;
+  uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+
+  const int STB = args.stages;  // weight tiles in flight (or resident)
+  const bool resident = args.b_resident != 0;
+  const uint32_t b_bytes = args.b_bytes;
+  uint8_t *sOp = smem;  // HALO: 2 halo buffers; GATHER: stages_a A tiles
+  uint8_t *sB = smem + args.off_b;
+  uint8_t *sG = smem + args.off_g;  // packed staging
+  uint8_t *sE = smem + args.off_e;  // epilogue byte rows
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + args.off_bar);
+  // barriers: full_b[STB] empty_b[STB] opfull[NO] opempty[NO] accfull[2] accempty[2] drain
+  //           ebar_full[4] ebar_free[4] (epilogue byte rows, per row quadrant)
+  const int NO = HALO ? 2 : args.stages_a;
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 2 * STB + 2 * NO + 13);
+  auto full_b = [&](int s) { return ptx::smem_addr(bars + s); };
+  auto empty_b = [&](int s) { return ptx::smem_addr(bars + STB + s); };
+  auto opfull = [&](int s) { return ptx::smem_addr(bars + 2 * STB + s); };
+  auto opempty = [&](int s) { return ptx::smem_addr(bars + 2 * STB + NO + s); };
+  auto accfull = [&](int a) { return ptx::smem_addr(bars + 2 * STB + 2 * NO + a); };
+  auto accempty = [&](int a) { return ptx::smem_addr(bars + 2 * STB + 2 * NO + 2 + a); };
+  const uint32_t drain_bar = ptx::smem_addr(bars + 2 * STB + 2 * NO + 4);
+  auto ebar_full = [&](int q) { return ptx::smem_addr(bars + 2 * STB + 2 * NO + 5 + q); };
+  auto ebar_free = [&](int q) { return ptx::smem_addr(bars + 2 * STB + 2 * NO + 9 + q); };
+
+  volatile int *status = args.status;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) s_skip = *status;
+  __syncthreads();
+  if (s_skip) return;
+  if (warp == 0) {
+    ptx::tmem_alloc(ptx::smem_addr(tmem_holder), args.tmem_cols);
+    ptx::tmem_relinquish();
+  }
+  if (threadIdx.x == 32) {
+    for (int s = 0; s < STB; ++s) {
+      ptx::mbar_init(full_b(s), 1);
+      ptx::mbar_init(empty_b(s), 1);
+    }
+    for (int s = 0; s < NO; ++s) {
+      ptx::mbar_init(opfull(s), HALO ? kProdWarps : kProdWarps / 2);
+      ptx::mbar_init(opempty(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      ptx::mbar_init(accfull(a), 1);
+      ptx::mbar_init(accempty(a), kEpiWarps);
+    }
+    ptx::mbar_init(drain_bar, 1);
+    for (int q = 0; q < 4; ++q) {
+      ptx::mbar_init(ebar_full(q), 1);
+      ptx::mbar_init(ebar_free(q), 1);
+    }
+    ptx::fence_barrier_init();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  const long long total_tiles = static_cast<long long>(args.grid_m) * args.nblocks;
+  const long long first_tile = blockIdx.x, tile_step = gridDim.x;
+  const int nchunks = args.nchunks;  // weight tiles per output tile
+  bool ok = true;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---- weight tiles ----
+      ptx::prefetch_tmap(&tmap_b);
+      if (resident) {
+        for (int c = 0; c < nchunks; ++c) {
+          ptx::mbar_arrive_expect_tx(full_b(c), b_bytes);
+          ptx::tma_load_2d(ptx::smem_addr(sB + c * b_bytes), &tmap_b, c * BK, 0, full_b(c));
+        }
+      } else {
+        long long cb = 0, issued_from = 0;
+        for (long long tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
+          const int nb = static_cast<int>(tile / args.grid_m);
+          for (int c = 0; c < nchunks; ++c, ++cb) {
+            const int s = static_cast<int>(cb % STB);
+            const long long round = cb / STB;
+            if (round > 0 &&
+                !ptx::mbar_wait_bounded(empty_b(s), static_cast<uint32_t>((round - 1) & 1), status, kWaitLimitNs)) {
+              ok = false;
+              break;
+            }
+            ptx::mbar_arrive_expect_tx(full_b(s), b_bytes);
+            ptx::tma_load_2d(ptx::smem_addr(sB + s * b_bytes), &tmap_b, c * BK, nb * args.mma_n, full_b(s));
+          }
+        }
+        if (!ok) {  // leave no copy in flight: wait (bounded) for the last ring's worth
+          for (long long k = (cb - STB > issued_from ? cb - STB : issued_from); k < cb; ++k)
+            ptx::mbar_wait_bounded(full_b(static_cast<int>(k % STB)), static_cast<uint32_t>((k / STB) & 1), status,
+                                   kWaitLimitNs / 10);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---- MMA issue ----
+    // The whole warp runs this loop on warp-uniform values and one elected
+    // lane (always the same one: all lanes are converged) issues each
+    // tcgen05.mma and tcgen05.commit. Running the loop in one thread alone
+    // turns every descriptor into a per-thread value that has to be moved to
+    // the uniform datapath before each MMA, which costs more than the MMA.
+    const uint32_t idesc = ptx::idesc_f16_f32(BM, args.mma_n);
+    auto wait = [&](uint32_t bar, uint32_t parity) {
+      bool w_ok = true;
+      if (lane == 0) w_ok = ptx::mbar_wait_bounded(bar, parity, status, kWaitLimitNs);
+      return __shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0) != 0;
+    };
+    // Ring positions advance by increments (no division in this loop).
+    int sb = 0, so = 0;
+    uint32_t bpar = 0, opar = 0;
+    const uint32_t sB_addr = ptx::smem_addr(sB), sOp_addr = ptx::smem_addr(sOp);
+    const int nops = HALO ? args.nck : nchunks;  // operand stages per tile
+    const int taps_here = HALO ? args.taps : 1;
+    constexpr uint32_t a_row16 = T::kRowBytes / 16;  // one operand row in descriptor units
+    const uint32_t a_skip16 = HALO ? static_cast<uint32_t>(args.row_step - args.S) * a_row16 : 0u;
+    if (resident)  // resident weights: wait for all of them once
+      for (int c = 0; c < nchunks && ok; ++c)
+        if (!wait(full_b(c), 0)) ok = false;
+    long long i = 0;
+    for (long long tile = first_tile; tile < total_tiles && ok; tile += tile_step, ++i) {
+      const int a = static_cast<int>(i & 1);
+      if (i >= 2 && !wait(accempty(a), static_cast<uint32_t>(((i >> 1) - 1) & 1))) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();  // the epilogue's reads of this accumulator are complete
+      const uint32_t tmem_d = tmem_base + static_cast<uint32_t>(a * args.mma_n);
+      uint32_t acc = 0;
+      for (int j = 0; j < nops && ok; ++j) {
+        if (!wait(opfull(so), opar)) {
+          ok = false;
+          break;
+        }
+        int words = (HALO ? args.wpr : args.words_total) - j * WC;
+        if (words > WC) words = WC;
+        const int ksteps = (words * U::L + T::kKPerMma - 1) / T::kKPerMma;
+        // No tcgen05 fence here: the operands arrived through the async proxy
+        // (TMA, or stores fenced with fence.proxy.async before the producers'
+        // arrive), which the mbarrier wait already orders.
+        const uint64_t a0 = T::desc(sOp_addr + so * args.op_stride);
+        if (resident) {
+          const uint64_t b0 = T::desc(sB_addr + (HALO ? j * taps_here : j) * b_bytes);
+          if (ptx::elect_one())
+            issue_taps<FP8>(tmem_d, a0, b0, idesc, ksteps, taps_here, args.S, a_row16, a_skip16, b_bytes >> 4, acc);
+          __syncwarp();
+          acc = 1;
+        } else {
+          uint64_t adesc = a0;
+          int ts = 0;
+          for (int t = 0; t < taps_here; ++t) {
+            if (!wait(full_b(sb), bpar)) {
+              ok = false;
+              break;
+            }
+            const uint64_t bdesc = T::desc(sB_addr + sb * b_bytes);
+            if (ptx::elect_one()) {
+              mma_ksteps<FP8>(ksteps, tmem_d, adesc, bdesc, idesc, acc);
+              ptx::mma_commit(empty_b(sb));
+            }
+            __syncwarp();
+            acc = 1;
+            if (++sb == STB) {
+              sb = 0;
+              bpar ^= 1;
+            }
+            if (HALO) {
+              adesc += a_row16;  // next halo row
+              if (++ts == args.S) {
+                ts = 0;
+                adesc += a_skip16;
+              }
+            }
+          }
+        }
+        if (ptx::elect_one()) ptx::mma_commit(opempty(so));  // the stage is free once these MMAs complete
+        __syncwarp();
+        if (++so == NO) {
+          so = 0;
+          opar ^= 1;
+        }
+      }
+      if (ok) {
+        if (ptx::elect_one()) ptx::mma_commit(accfull(a));
+        __syncwarp();
+      }
+    }
+    if (ptx::elect_one()) ptx::mma_commit(drain_bar);
+    __syncwarp();
+    if (lane == 0) {
+      int quiet = 0;
+      ptx::mbar_wait_bounded(drain_bar, 0, &quiet, kWaitLimitNs);
+    }
+    __syncwarp();
+  } else if (warp < kFirstEpiWarp) {
+    // ---- operand producers ----
+    const int t = threadIdx.x - 64;  // 0 .. kProdThreads - 1
+    const W *act = static_cast<const W *>(args.act);
+    auto wait_lane0 = [&](uint32_t bar, uint32_t parity) {
+      bool w_ok = true;
+      if (lane == 0) w_ok = ptx::mbar_wait_bounded(bar, parity, status, kWaitLimitNs);
+      return __shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0) != 0;
+    };
+    if constexpr (HALO) {
+      const int halo_rows = args.nseg * args.seg_rows;
+      // halo row hr -> virtual offset from the tile's first position, or -1
+      auto voff = [&](int hr) -> int {
+        const int g = static_cast<int>(fdiv(static_cast<uint32_t>(hr), args.fd_seg));
+        const int q = hr - g * args.seg_rows;
+        return q < args.seg_used ? g * args.Wp + q : -1;
+      };
+      // items k = (tile i, channel chunk j), in the MMA's order
+      auto gather = [&](long long tile, int j, int slot) {
+        const uint32_t mt = static_cast<uint32_t>(tile) - fdiv(static_cast<uint32_t>(tile), args.fd_gm) * args.fd_gm.d;
+        const uint32_t v0 = mt * BM;
+        const uint32_t dst0 = ptx::smem_addr(sG + slot * args.g_stride);
+        for (int hr = t; hr < halo_rows; hr += kProdThreads) {
+          const int off = voff(hr);
+          if (off < 0) continue;
+          const uint32_t u = v0 + static_cast<uint32_t>(off);
+          const uint32_t img = fdiv(u, args.fd_plane);
+          const uint32_t rem = u - img * args.fd_plane.d;
+          const uint32_t ihp = fdiv(rem, args.fd_wp);
+          const int ih = static_cast<int>(ihp) - args.pad;
+          const int iw = static_cast<int>(rem - ihp * args.fd_wp.d) - args.pad;
+          const bool valid = static_cast<int>(img) < args.N && ih >= 0 && ih < args.H && iw >= 0 && iw < args.W;
+          const W *px = act + ((static_cast<long long>(img) * args.H + ih) * args.W + iw) * args.wpr + j * WC;
+          const uint32_t dst = dst0 + hr * St::kRowBytes;
+          if (args.gather_vec) {
+            stage_chunk<W, WC>(dst, reinterpret_cast<const char *>(valid ? px : act), valid ? 1u : 0u);
+          } else {
+#pragma unroll
+            for (int q = 0; q < WC; ++q) {
+              const bool in = valid && j * WC + q < args.wpr;
+              const W *src = in ? px + q : act;
+              if constexpr (sizeof(W) == 8)
+                ptx::cp_async_8(dst + 8 * q, src, in ? 8u : 0u);
+              else
+                ptx::cp_async_4(dst + 4 * q, src, in ? 4u : 0u);
+            }
+          }
+        }
+      };
+      long long ntile = first_tile;
+      int nj = 0;
+      auto advance = [&](long long &tile, int &j) {
+        if (++j == args.nck) {
+          j = 0;
+          tile += tile_step;
+        }
+      };
+      if (ntile < total_tiles) gather(ntile, nj, 0);
+      ptx::cp_async_commit();
+      long long ctile = ntile;
+      advance(ntile, nj);
+      for (long long k = 0; ctile < total_tiles; ++k) {
+        if (ntile < total_tiles) gather(ntile, nj, static_cast<int>((k + 1) & 1));
+        ptx::cp_async_commit();
+        ptx::cp_async_wait<1>();  // item k of this thread's rows has landed
+        const int hb = static_cast<int>(k & 1);
+        if (k >= 2 && !wait_lane0(opempty(hb), static_cast<uint32_t>(((k >> 1) - 1) & 1))) {
+          ok = false;
+          break;
+        }
+        const uint8_t *stg = sG + hb * args.g_stride;
+        for (int hr = t; hr < halo_rows; hr += kProdThreads) {
+          if (voff(hr) < 0) continue;  // a row no tap reads
+          W cur[WC];
+          load_staged<W, WC>(stg + hr * St::kRowBytes, cur);
+          U::unpack_row(cur, sOp + hb * args.op_stride, hr);
+        }
+        ptx::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(opfull(hb));
+        ctile = ntile;
+        advance(ntile, nj);
+      }
+      ptx::cp_async_wait<0>();
+    } else {
+      // GATHER: group grp (four warps) takes items grp, grp + 2, ...; thread
+      // row of the group owns row `row` of every A tile it fills
+      const int grp = t / BM, row = t % BM;
+      AGather<W, WC> g;
+      g.act = act;
+      g.H = args.H;
+      g.W_ = args.W;
+      g.wpr = args.wpr;
+      g.S = args.S;
+      g.stride = args.stride;
+      g.pad = args.pad;
+      g.words_total = args.words_total;
+      g.vec = args.gather_vec != 0;
+      auto set_tile = [&](long long tile) {
+        const uint32_t tl = static_cast<uint32_t>(tile);
+        const uint32_t mt = tl - fdiv(tl, args.fd_gm) * args.fd_gm.d;
+        const uint32_t m = mt * BM + row;
+        g.row_valid = m < static_cast<uint64_t>(args.M);
+        const uint32_t mm = g.row_valid ? m : 0u;
+        const uint32_t tq = fdiv(mm, args.fd_wo);
+        g.ow = static_cast<int>(mm - tq * args.fd_wo.d);
+        const uint32_t nq = fdiv(tq, args.fd_ho);
+        g.oh = static_cast<int>(tq - nq * args.fd_ho.d);
+        g.n = static_cast<int>(nq);
+      };
+      constexpr uint32_t kSlotBytes = BM * St::kRowBytes;
+      const uint32_t slot0 = ptx::smem_addr(sG) + grp * (kGatherDepth * kSlotBytes) + row * St::kRowBytes;
+      // issue side: this group's item (itile, ic), kGatherDepth ahead of the consume side
+      long long itile = first_tile;
+      int ic = 0;
+      auto step = [&]() {
+        if (++ic == nchunks) {
+          ic = 0;
+          itile += tile_step;
+        }
+      };
+      if (grp == 1) step();
+      if (itile < total_tiles) set_tile(itile);
+      auto issue_next = [&](int slot) {
+        if (itile < total_tiles) {
+          g.issue(ic, slot0 + slot * kSlotBytes);
+          const long long prev = itile;
+          step();
+          step();
+          if (itile != prev && itile < total_tiles) set_tile(itile);
+        }
+        ptx::cp_async_commit();
+      };
+#pragma unroll 1
+      for (int d = 0; d < kGatherDepth; ++d) issue_next(d);
+      const long long items = ((total_tiles - first_tile + tile_step - 1) / tile_step) * nchunks;
+      int slot = 0;
+      for (long long k = grp; k < items; k += 2) {
+        ptx::cp_async_wait<kGatherDepth - 1>();
+        W cur[WC];
+        load_staged<W, WC>(sG + grp * (kGatherDepth * kSlotBytes) + slot * kSlotBytes + row * St::kRowBytes, cur);
+        const int sa = static_cast<int>(k % NO);
+        const long long round = k / NO;
+        if (round > 0 && !wait_lane0(opempty(sa), static_cast<uint32_t>((round - 1) & 1))) {
+          ok = false;
+          break;
+        }
+        U::unpack_row(cur, sOp + sa * args.op_stride, row);
+        ptx::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) ptx::mbar_arrive(opfull(sa));
+        issue_next(slot);  // refill the slot just read
+        if (++slot == kGatherDepth) slot = 0;
+      }
+      ptx::cp_async_wait<0>();
+    }
+  } else {
+    // ---- epilogue ----
+    const int quad = warp & 3;
+    const int half = (warp - kFirstEpiWarp) / 4;
+    const int row = quad * 32 + lane;
+    long long i = 0;
+    for (long long tile = first_tile; tile < total_tiles; tile += tile_step, ++i) {
+      const int a = static_cast<int>(i & 1);
+      bool w_ok = true;
+      if (lane == 0) w_ok = ptx::mbar_wait_bounded(accfull(a), static_cast<uint32_t>((i >> 1) & 1), status, kWaitLimitNs);
+      if (!__shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0)) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();
+      const uint32_t tl = static_cast<uint32_t>(tile);
+      const uint32_t nbu = fdiv(tl, args.fd_gm);
+      const int nb = static_cast<int>(nbu);
+      const uint32_t mt = tl - nbu * args.fd_gm.d;
+      bool valid;
+      long long m;
+      if (HALO) {
+        const uint32_t v = mt * BM + row;
+        const uint32_t img = fdiv(v, args.fd_plane);
+        const uint32_t rem = v - img * args.fd_plane.d;
+        const uint32_t oh = fdiv(rem, args.fd_wp);
+        const uint32_t ow = rem - oh * args.fd_wp.d;
+        valid = static_cast<int>(img) < args.N && static_cast<int>(oh) < args.Ho && static_cast<int>(ow) < args.Wo;
+        m = (static_cast<long long>(img) * args.Ho + oh) * args.Wo + ow;
+      } else {
+        m = static_cast<long long>(mt) * BM + row;
+        valid = m < args.M;
+      }
+      const uint32_t taddr = tmem_base + static_cast<uint32_t>(a * args.mma_n) + (static_cast<uint32_t>(quad * 32) << 16);
+      if (!epilogue_row(args, taddr, valid, m, nb, sE, row, half, ebar_full(quad), ebar_free(quad), i)) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(accempty(a));
+    }
+  }
+
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem_base, args.tmem_cols);
+  }
+  if (!ok) atomicOr(const_cast<int *>(status), static_cast<int>(SAMD_ETIMEOUT));
+}
+
+// cudaFuncSetAttribute once per (kernel, device); defined in conv2d.cu.
+cudaError_t ensure_smem_attr(const void *kern, size_t smem);
+
+template <typename W, int BITS, bool SIGNED, bool FP8>
+cudaError_t launch_conv(const CUtensorMap &tmap, const ConvArgs &args, bool halo, dim3 grid, size_t smem,
+                        cudaStream_t s) {
+  auto kern = halo ? conv_kernel<W, BITS, SIGNED, true, FP8> : conv_kernel<W, BITS, SIGNED, false, FP8>;
+  cudaError_t e = ensure_smem_attr(reinterpret_cast<const void *>(kern), smem);
+  if (e != cudaSuccess) return e;
+  kern<<<grid, kThreads, smem, s>>>(tmap, args);
+  return cudaGetLastError();
+}
+
+// Launchers by operand type, word width and lane width (one translation unit
+// each, so that they compile in parallel).
+#define SAMD_CONV_LAUNCHER(name)                                                                             \
+  cudaError_t name(int bits, bool is_signed, const CUtensorMap &tmap, const ConvArgs &args, bool halo, dim3 grid, \
+                   size_t smem, cudaStream_t s);
+SAMD_CONV_LAUNCHER(launch_conv_f16_w32a)  // 1-4-bit lanes
+SAMD_CONV_LAUNCHER(launch_conv_f16_w32b)  // 5-8-bit lanes
+SAMD_CONV_LAUNCHER(launch_conv_f16_w64)
+SAMD_CONV_LAUNCHER(launch_conv_f8_w32)
+SAMD_CONV_LAUNCHER(launch_conv_f8_w64)
+#undef SAMD_CONV_LAUNCHER
+
+}  // namespace conv
+}  // namespace samd

@@ -61,6 +61,15 @@ __device__ __forceinline__ bool mbar_try_wait_hint(uint32_t bar, uint32_t parity
   return ok != 0;
 }
 
+// One lane of a converged warp (the same lane every time) gets true.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t pred = 0;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\telect.sync _|p, 0xffffffff;\n\tselp.u32 %0, 1, 0, p;\n}"
+      : "=r"(pred));
+  return pred != 0;
+}
+
 // Wait for the phase with the given parity to complete. Gives up after
 // `limit_ns` of wall time, or as soon as another CTA has recorded a failure
 // in *status; either way it returns false and the caller stops its work.
@@ -139,6 +148,19 @@ __device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t a_desc, uint64
       : "memory");
 }
 
+// D[tmem] (+)= A * B^T with e4m3 A and B (K = 32), fp32 accumulation. The
+// e4m3 format code is 0 in the descriptor, as fp16 is for kind::f16, so the
+// same instruction descriptor serves both kinds.
+__device__ __forceinline__ void mma_f8(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                       uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 // Arrive once on `bar` when every tcgen05 op issued so far by this thread completes.
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
@@ -170,6 +192,18 @@ __device__ __forceinline__ uint64_t sw128_kmajor_desc(uint32_t saddr) {
   d |= static_cast<uint64_t>(1024 >> 4) << 32;         // stride byte offset: next 8-row group
   d |= static_cast<uint64_t>(1) << 46;                 // descriptor version for tcgen05
   d |= static_cast<uint64_t>(2) << 61;                 // swizzle mode: 128-byte
+  return d;
+}
+
+// The same for 64-byte rows with the 64-byte swizzle (8-row groups of 512
+// bytes): chunk c of row r is stored at chunk c ^ ((r / 2) % 4).
+__device__ __forceinline__ uint64_t sw64_kmajor_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+  d |= static_cast<uint64_t>(1) << 16;
+  d |= static_cast<uint64_t>(512 >> 4) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(4) << 61;  // swizzle mode: 64-byte
   return d;
 }
 
