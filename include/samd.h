@@ -154,11 +154,17 @@ typedef struct {
  * workspace / workspace_bytes: caller-owned device scratch of at least
  * samd_conv2d_workspace_size(...) bytes (16-byte aligned) that receives the
  * weights in the tensor-core operand layout on every call.
- * Exactness: the sum runs on the tensor cores over fp16 operands with fp32
- * accumulation, exact while every partial sum stays below 2^24. If
+ * Exactness: the sum runs on the tensor cores with fp32 accumulation, exact
+ * while every partial sum stays below 2^24, over e4m3 operands when
+ * max|a| <= 16 and max|w| <= 16 (lanes of up to 4 bits, and signed 5-bit
+ * lanes: every such integer is exact in e4m3) and over fp16 operands
+ * otherwise (samd_conv2d_operand_bits tells which). If
  * R*S*C * max|a| * max|w| reaches 2^24 and the weights have 5-8 bits, the
  * weights are split into two 4-bit digits (two exact accumulators per
  * output); if R*S*C * max|a| * 16 also reaches 2^24, SAMD_EUNSUP.
+ * Scheduling: a layer of fewer than 4 x (SM count) 128-pixel tiles runs on
+ * ceil(tiles / 4) SMs, so that independent layers issued on other streams
+ * run beside it.
  * Other limits (SAMD_EUNSUP): spacer 0 for fa and fw; R, S <= 16.
  * A kernel that gives up on a bounded wait leaves its outputs undefined and
  * records SAMD_ETIMEOUT for samd_device_status.
@@ -171,6 +177,11 @@ SAMD_API samd_status samd_conv2d(const samd_conv_desc *desc, samd_fmt fa, const 
  * output format (0 on error). The same size suffices for
  * samd_conv2d_prepare. */
 SAMD_API size_t samd_conv2d_workspace_size(const samd_conv_desc *desc, samd_fmt fa, samd_fmt fw);
+
+/* Width in bits of the tensor-core operands samd_conv2d uses for this shape
+ * and these formats: 8 (e4m3), 16 (fp16), or 0 if the convolution is
+ * rejected (invalid arguments or SAMD_EUNSUP). Host-only; no GPU needed. */
+SAMD_API int samd_conv2d_operand_bits(const samd_conv_desc *desc, samd_fmt fa, samd_fmt fw);
 
 /*
  * Weights prepared once, used by many calls (the weights of an inference

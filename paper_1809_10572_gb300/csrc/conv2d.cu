@@ -62,7 +62,7 @@ namespace {
 struct WPrepArgs {
   int K, C, RS;
   int bits_w, signed_w, lane_w_w, Lw, wpr_w;  // weight format
-  int bits_a, La, WC, wpr_a, words_total;      // reduction order set by the activation format
+  int bits_a, signed_a, fp8, La, WC, wpr_a, words_total;  // reduction order set by the activation format
   int Kpad, n_mma, mma_n, NBc, split;
   int halo, taps;  // halo: reduction order (chunk, tap, position); else (tap-major words, position)
   long long rows_total;
@@ -107,7 +107,7 @@ __global__ void __launch_bounds__(256) wprep_kernel(const WW *__restrict__ wt, v
         wi = kw % a.wpr_a;
       }
       if (kw < a.words_total) {
-        const int ch = wi * a.La + kpos_lane(a.bits_a, pos);
+        const int ch = wi * a.La + kpos_lane_op(a.bits_a, a.signed_a != 0, a.fp8 != 0, pos);
         if (ch < a.C) {
           const long long wrow = static_cast<long long>(k) * a.RS + tap;
           const WW word = wt[wrow * a.wpr_w + ch / a.Lw];
@@ -154,6 +154,7 @@ struct Plan {
   long long grid_m;                        // 128-position tiles along the output
   int stages_a, b_resident;
   long long M;
+  long long bound;  // R*S*C * max|a| * max|w|: no accumulator exceeds it
   uint32_t tmem_cols;
   uint32_t op_stride, off_b, b_bytes, off_g, g_stride, off_e, off_bar;
   size_t smem_bytes;
@@ -165,6 +166,7 @@ long long max_abs(samd_fmt f) { return f.is_signed ? (1LL << (f.bits - 1)) : ((1
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 constexpr int kMaxHaloRows = 640;
+constexpr int kMinTilesPerCta = 4;
 
 // Tiling, reduction order, operand type and exactness mode for one
 // convolution. fo.bits == 0 means no packed output. Returns SAMD_EUNSUP when
@@ -174,6 +176,7 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
   if (p.La == 0) return SAMD_EINVAL;
   const long long taps = static_cast<long long>(d->R) * d->S * d->C;
   const long long bound = taps * max_abs(fa) * max_abs(fw);
+  p.bound = bound;
   p.split = 0;
   if (bound >= (1LL << 24)) {
     // two 4-bit weight digits: each accumulator sums at most taps * max|a| * 16
@@ -211,14 +214,12 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
   p.gather_vec = (p.wpr % p.WC == 0) && ((static_cast<long long>(p.wpr) * wb) % vec == 0) ? 1 : 0;
   p.b_bytes = static_cast<uint32_t>(p.mma_n) * p.row_bytes;  // a multiple of 1024
   const size_t bst = p.b_bytes;
-  const bool fast_out = fo.bits != 0 && (fo.word_bits == 32 ? (32 % lanes_per_word(fo) == 0 && lanes_per_word(fo) >= 4)
-                                                            : (32 % lanes_per_word(fo) == 0 && lanes_per_word(fo) >= 8));
-  const size_t e_bytes = (fo.bits == 0 || fast_out) ? 0 : round_up(BM * ((p.n_mma + 31) / 32 * 32 + 4), 16);
+  const size_t e_bytes = 0;  // the epilogue packs in registers
   // mbarriers: full_b and empty_b per weight stage, opfull and opempty per
-  // operand stage, two accumulator pairs, the drain barrier and two per
-  // epilogue row quadrant; then the TMEM address word
+  // operand stage, two accumulator pairs and the drain barrier; then the
+  // TMEM address word
   auto bar_bytes = [](int stages, int op_stages) {
-    return round_up(static_cast<size_t>(2 * stages + 2 * op_stages + 13) * 8 + 4, 16);
+    return round_up(static_cast<size_t>(2 * stages + 2 * op_stages + 5) * 8 + 4, 16);
   };
   const size_t kBudget = 224 * 1024;  // below the 227 KB opt-in limit minus static shared memory
   auto finish = [&](size_t op_bytes, size_t g_bytes, int op_stages) {
@@ -314,7 +315,7 @@ samd_fmt none_fmt() { return samd_fmt{0, 0, 0, 0}; }
 bool layout_ok(const Plan &p) {
   const size_t NO = p.halo ? 2 : static_cast<size_t>(p.stages_a);
   const size_t op_bytes = NO * p.op_stride;
-  const size_t bars = (2 * static_cast<size_t>(p.stages) + 2 * NO + 13) * 8 + 4;
+  const size_t bars = (2 * static_cast<size_t>(p.stages) + 2 * NO + 5) * 8 + 4;
   return p.stages >= 1 && NO >= 2 && op_bytes <= p.off_b &&
          p.off_b + static_cast<size_t>(p.stages) * p.b_bytes <= p.off_g && p.off_g + 2 * p.g_stride <= p.off_e &&
          p.off_e <= p.off_bar && 1023 + p.off_bar + bars <= p.smem_bytes && p.op_stride % 1024 == 0 &&
@@ -363,6 +364,12 @@ size_t conv2d_workspace_size(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw) 
   return best;
 }
 
+int conv2d_operand_bits(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw) {
+  conv::Plan p;
+  if (conv::make_plan(d, fa, fw, conv::none_fmt(), p) != SAMD_OK) return 0;
+  return p.fp8 ? 8 : 16;
+}
+
 samd_status conv2d_check(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw) {
   conv::Plan p;
   return conv::make_plan(d, fa, fw, conv::none_fmt(), p);
@@ -385,6 +392,8 @@ samd_status conv2d_prepare(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, co
   wa.Lw = lanes_per_word(fw);
   wa.wpr_w = static_cast<int>(words_per_row(fw, d->C));
   wa.bits_a = fa.bits;
+  wa.signed_a = fa.is_signed;
+  wa.fp8 = p.fp8;
   wa.La = p.La;
   wa.WC = p.WC;
   wa.wpr_a = p.wpr;
@@ -487,6 +496,9 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
     a.out_fast = fast ? Lo : 0;
   }
   a.shift = shift;
+  a.out_scale = ldexpf(1.0f, -shift);
+  a.fast_req = (!p.split && (p.bound >> shift) < (1LL << 22)) ? 1 : 0;
+  a.fast_acc = (!p.split && p.bound < (1LL << 22)) ? 1 : 0;
   a.Hv = p.Hv;
   a.Wp = p.Wp;
   a.nseg = p.nseg;
@@ -513,9 +525,11 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   a.g_stride = p.g_stride;
   a.off_e = p.off_e;
   a.off_bar = p.off_bar;
+  // a small layer keeps at least kMinTilesPerCta tiles per CTA, leaving SMs
+  // to independent layers issued on other streams
   const long long total_tiles = p.grid_m * p.nblocks;
-  long long ctas = sm_count();
-  if (ctas > total_tiles) ctas = total_tiles;
+  long long ctas = (total_tiles + kMinTilesPerCta - 1) / kMinTilesPerCta;
+  if (ctas > sm_count()) ctas = sm_count();
   dim3 grid(static_cast<unsigned>(ctas));
   const bool halo = p.halo != 0;
   cudaError_t e;

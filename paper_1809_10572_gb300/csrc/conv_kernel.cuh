@@ -75,6 +75,47 @@ __host__ __device__ constexpr int kpos_lane(int bits, int pos) {
   return pos;
 }
 
+// e4m3 widening by byte permutes (1- and 2-bit lanes, unsigned 4-bit lanes):
+// each lane of a 32-bit half-word becomes a selector nibble of prmt over a
+// table of e4m3 codes. The reduction positions of such a half-word are
+// ordered by how the nibbles are formed (identity for 4 bits; even then odd
+// lanes for 2 bits; lanes k, k+4, ... for 1 bit); A and B use the same order.
+__host__ __device__ constexpr bool prmt8(int bits, bool is_signed) {
+  return bits == 1 || bits == 2 || (bits == 4 && !is_signed);
+}
+__host__ __device__ constexpr int kpos_lane_prmt32(int bits, int p) {
+  return bits == 4 ? p : (bits == 2 ? 2 * (p % 4 + 4 * ((p / 4) % 2)) + p / 8 : 4 * (p % 8) + p / 8);
+}
+// The lane of an activation word held by reduction position `pos` for the
+// operand type in use.
+__host__ __device__ constexpr int kpos_lane_op(int bits, bool is_signed, bool fp8, int pos) {
+  return (fp8 && prmt8(bits, is_signed)) ? (pos / (32 / bits)) * (32 / bits) + kpos_lane_prmt32(bits, pos % (32 / bits))
+                                         : kpos_lane(bits, pos);
+}
+
+// e4m3 code of a small integer (|v| <= 16): sign, exponent biased by 7, three
+// mantissa bits.
+__host__ __device__ constexpr uint32_t e4m3_code(int v) {
+  if (v == 0) return 0u;
+  const uint32_t sign = v < 0 ? 0x80u : 0u;
+  const int a = v < 0 ? -v : v;
+  int e = 0;
+  while ((a >> (e + 1)) != 0) ++e;
+  return sign | static_cast<uint32_t>((e + 7) << 3) | static_cast<uint32_t>(((a << 3) >> e) - 8);
+}
+__host__ __device__ constexpr uint32_t e4m3_table4(int v0, int v1, int v2, int v3) {
+  return e4m3_code(v0) | (e4m3_code(v1) << 8) | (e4m3_code(v2) << 16) | (e4m3_code(v3) << 24);
+}
+
+// prmt.b32 in its default mode: byte i of the result is byte (c_i & 7) of
+// {b, a}, or, when bit 3 of selector nibble c_i is set, that byte's sign bit
+// repeated eight times.
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t c) {
+  uint32_t d;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
+
 // n / d for 0 <= n < 2^31 by one multiply-high, an add and a shift:
 // l = ceil(log2 d), m = floor(2^32 (2^l - d) / d) + 1, q = (umulhi(m, n) + n) >> l.
 struct FastDiv {
@@ -114,8 +155,11 @@ struct ConvArgs {
   int gather_vec;   // AGather::vec
   uint32_t tmem_cols;
   int out_bits, out_signed, out_lane_w, out_L, out_word64, out_wpr;
-  int out_fast;     // output lanes per word when they divide 32 (packing in registers), else 0
+  int out_fast;     // output lanes per word when they divide 32 (whole words per 32 channels), else 0
   int shift;
+  float out_scale;  // 2^-shift
+  int fast_req;     // |acc| / 2^shift < 2^22: requantize through floor_scaled_biased
+  int fast_acc;     // |acc| < 2^22: int32 outputs through floor_scaled_biased
   // HALO (stride 1): virtual output grid of N x Hv x Wp positions. A tile of
   // 128 consecutive positions v0.. reads nseg segments of the input grid:
   // segment g holds seg_used rows starting at virtual row v0 + g * Wp and
@@ -198,10 +242,55 @@ struct AUnpack {
     ((h[P] = pair<P>(w)), ...);
   }
 
+  static constexpr bool kPrmt = FP8 && prmt8(BITS, SIGNED);
+
+  // The e4m3 bytes of the lanes of one 32-bit half-word, in reduction order
+  // (32 / BITS bytes into out[0 .. 8 / BITS)).
+  __device__ static __forceinline__ void prmt_half(uint32_t x, uint32_t *out) {
+    if constexpr (BITS == 4) {
+      // nibbles 0-7 select e(0..7); nibbles 8-15 select the sign (0) of that
+      // table and, with bit 3 flipped, e(8..15) from the other one
+      constexpr uint32_t t0 = e4m3_table4(0, 1, 2, 3), t1 = e4m3_table4(4, 5, 6, 7);
+      constexpr uint32_t t2 = e4m3_table4(8, 9, 10, 11), t3 = e4m3_table4(12, 13, 14, 15);
+      const uint32_t xx = x ^ 0x88888888u;
+      out[0] = prmt(t0, t1, x) | prmt(t2, t3, xx);
+      out[1] = prmt(t0, t1, x >> 16) | prmt(t2, t3, xx >> 16);
+    } else if constexpr (BITS == 2) {
+      constexpr uint32_t t = SIGNED ? e4m3_table4(0, 1, -2, -1) : e4m3_table4(0, 1, 2, 3);
+      const uint32_t se = x & 0x33333333u, so = (x >> 2) & 0x33333333u;
+      out[0] = prmt(t, 0u, se);
+      out[1] = prmt(t, 0u, se >> 16);
+      out[2] = prmt(t, 0u, so);
+      out[3] = prmt(t, 0u, so >> 16);
+    } else {
+      constexpr uint32_t t = SIGNED ? e4m3_table4(0, -1, 0, 0) : e4m3_table4(0, 1, 0, 0);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t sk = (x >> k) & 0x11111111u;
+        out[2 * k] = prmt(t, 0u, sk);
+        out[2 * k + 1] = prmt(t, 0u, sk >> 16);
+      }
+    }
+  }
+
   // Widen one pixel's chunk and store it as row `row` of a swizzled K-major
   // operand whose rows are OpTraits::kRowBytes apart.
   __device__ static __forceinline__ void unpack_row(W (&w)[WC], uint8_t *tile, int row) {
     using T = OpTraits<FP8>;
+    if constexpr (kPrmt) {
+      constexpr int kHalves = WB / 32, kPer = 8 / BITS;  // 32-bit words of e4m3 bytes per half-word
+      uint32_t b[16];
+#pragma unroll
+      for (int q = 0; q < WC; ++q)
+#pragma unroll
+        for (int hh = 0; hh < kHalves; ++hh)
+          prmt_half(static_cast<uint32_t>(w[q] >> (32 * hh)), b + (q * kHalves + hh) * kPer);
+      uint8_t *rp = tile + row * T::kRowBytes;
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+        *reinterpret_cast<uint4 *>(rp + (T::swz(row, c) << 4)) = make_uint4(b[4 * c], b[4 * c + 1], b[4 * c + 2], b[4 * c + 3]);
+      return;
+    }
     if constexpr (SIGNED) {
 #pragma unroll
       for (int q = 0; q < WC; ++q) w[q] ^= sign_mask();
@@ -347,131 +436,252 @@ __device__ __forceinline__ void pack_regs(const uint32_t (&y)[32], int lane_w, i
   }
 }
 
-// Epilogue of one accumulator row (one output pixel m) of channel block nb,
-// for the 32-column groups g = half, half + 2, ...: fp32 accumulators ->
-// exact int32 -> optional int32 store, optional requantize-and-pack. Called
-// by whole warps (tcgen05.ld is collective). Output formats whose words do
-// not divide a 32-channel group go through one byte per channel in `ebuf`
-// (128 rows x ebytes): half 1 writes its bytes and arrives on `ebar_full`,
-// half 0 waits for it, assembles the row's words and arrives on `ebar_free`,
-// which half 1 awaits before it writes the next tile's bytes (tile index i).
-// Returns false when a bounded wait gave up.
-__device__ __forceinline__ bool epilogue_row(const ConvArgs &args, uint32_t taddr, bool row_valid, long long m,
-                                             int nb, uint8_t *ebuf, int row, int half, uint32_t ebar_full,
-                                             uint32_t ebar_free, long long i) {
-  const int lane = threadIdx.x & 31;
+constexpr int32_t kMagicBits = 0x4B400000;  // encoding of 1.5 * 2^23
+
+// floor(acc * scale) + 1.5 * 2^23 as the encoding of a float: with rounding
+// toward minus infinity the fma result, which lies in [2^23, 2^24) where the
+// unit in the last place is 1, is exactly floor(acc * scale) + 1.5 * 2^23
+// while |acc * scale| < 2^22 (scale = 2^-shift makes acc * scale exact).
+// The encoding is then kMagicBits + floor(acc * scale), monotonic in it.
+__device__ __forceinline__ int32_t floor_scaled_biased(float acc, float scale) {
+  float r;
+  asm("fma.rm.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(acc), "f"(scale), "f"(12582912.0f));
+  return __float_as_int(r);
+}
+
+// Packs lane patterns into words of L lanes one channel at a time (any L):
+// the running word `cur` receives lane nl at bit sh and is stored when full.
+template <typename WO>
+struct RowPacker {
+  WO *dst;
+  WO cur = 0;
+  int nl = 0, sh = 0;
+  __device__ __forceinline__ void put(uint32_t y, int L, int lw) {
+    cur |= static_cast<WO>(y) << sh;
+    sh += lw;
+    if (++nl == L) {
+      *dst++ = cur;
+      cur = 0;
+      sh = 0;
+      nl = 0;
+    }
+  }
+  __device__ __forceinline__ void flush() {
+    if (nl) *dst = cur;
+  }
+};
+
+// Epilogue of one accumulator row (one output pixel m) of channel block nb:
+// fp32 accumulators -> exact integers -> optional int32 store, optional
+// requantize-and-pack. Called by whole warps (tcgen05.ld is collective; rows
+// outside the output only skip the stores).
+//
+// The common case (packed output only, no split digits, |acc| / 2^shift <
+// 2^22) requantizes each accumulator with one fma in place.
+template <typename WO>
+__device__ __forceinline__ void epilogue_row_fast(const ConvArgs &args, uint32_t taddr, bool row_valid, long long m,
+                                                  int nb) {
+  const int ch0 = nb * args.NBc;
+  const int nvalid = args.K - ch0 < args.NBc ? args.K - ch0 : args.NBc;
+  const int lo = lane_lo(args.out_bits, args.out_signed), hi = lane_hi(args.out_bits, args.out_signed);
+  const int32_t blo = kMagicBits + lo, bhi = kMagicBits + hi;
+  const uint32_t omask = (1u << args.out_bits) - 1;
+  const float scale = args.out_scale;
+  const int L = args.out_L, lw = args.out_lane_w;
+  RowPacker<WO> pk;
+  pk.dst = static_cast<WO *>(args.packed_out) + (m * args.out_wpr + ch0 / L);
+  for (int col = 0; col < nvalid; col += 32) {
+    uint32_t y[32];
+    ptx::tmem_ld_32x32b_x32(taddr + col, y);
+    ptx::tmem_wait_ld();
+    const int cnt = nvalid - col < 32 ? nvalid - col : 32;
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      int32_t t = floor_scaled_biased(__uint_as_float(y[k]), scale);
+      t = t < blo ? blo : (t > bhi ? bhi : t);
+      y[k] = k < cnt ? static_cast<uint32_t>(t) & omask : 0u;
+    }
+    if (!row_valid) continue;
+    if (args.out_fast) {  // L divides 32: whole words per 32-channel group
+      WO *dst = static_cast<WO *>(args.packed_out) + (m * args.out_wpr + (ch0 + col) / L);
+      switch (args.out_fast) {
+        case 4:
+          if constexpr (sizeof(WO) == 4) pack_regs<4>(y, lw, cnt, dst);
+          break;
+        case 8: pack_regs<8>(y, lw, cnt, dst); break;
+        case 16: pack_regs<16>(y, lw, cnt, dst); break;
+        default: pack_regs<32>(y, lw, cnt, dst); break;
+      }
+    } else {
+#pragma unroll
+      for (int k = 0; k < 32; ++k)
+        if (k < cnt) pk.put(y[k], L, lw);
+    }
+  }
+  if (!args.out_fast && row_valid) pk.flush();
+}
+
+// The fast epilogue for output lanes of OB = 1, 2, 4 or 8 bits without
+// spacers: the words of a 32-channel group are built 32 bits at a time
+// (a 64-bit word is its two 32-bit halves, low half first, so the bytes are
+// the same) with compile-time shifts. Unsigned lanes are summed in the
+// biased domain and the bias sum is removed once per word; signed lanes are
+// masked to their two's complement bits first.
+template <int OB, bool OS>
+__device__ __forceinline__ void epilogue_row_spec(const ConvArgs &args, uint32_t taddr, bool row_valid, long long m,
+                                                  int nb) {
+  constexpr int LH = 32 / OB;  // lanes per 32-bit half-word
+  constexpr int NH = OB;       // half-words per 32-channel group
+  constexpr int32_t lo = OS ? -(1 << (OB - 1)) : 0, hi = OS ? (1 << (OB - 1)) - 1 : (1 << OB) - 1;
+  constexpr int32_t blo = kMagicBits + lo, bhi = kMagicBits + hi;
+  constexpr uint32_t omask = (1u << OB) - 1;
+  constexpr uint32_t bias_sum = [] {
+    uint32_t b = 0;
+    for (int l = 0; l < LH; ++l) b += static_cast<uint32_t>(kMagicBits) << (l * OB);
+    return b;
+  }();
+  const int ch0 = nb * args.NBc;
+  const int nvalid = args.K - ch0 < args.NBc ? args.K - ch0 : args.NBc;
+  const float scale = args.out_scale;
+  // 32-bit half-words of this row: output channel c sits in half-word c / LH
+  uint32_t *row32 = reinterpret_cast<uint32_t *>(static_cast<uint8_t *>(args.packed_out) +
+                                                 static_cast<size_t>(m) * args.out_wpr * (args.out_word64 ? 8 : 4)) +
+                    ch0 / LH;
+  for (int col = 0; col < nvalid; col += 32) {
+    uint32_t r[32];
+    ptx::tmem_ld_32x32b_x32(taddr + col, r);
+    ptx::tmem_wait_ld();
+    const int cnt = nvalid - col < 32 ? nvalid - col : 32;
+    uint32_t h[NH];
+#pragma unroll
+    for (int j = 0; j < NH; ++j) {
+      uint32_t w = 0;
+#pragma unroll
+      for (int l = 0; l < LH; ++l) {
+        int32_t t = floor_scaled_biased(__uint_as_float(r[j * LH + l]), scale);
+        t = t < blo ? blo : (t > bhi ? bhi : t);
+        if constexpr (OS)
+          w |= (static_cast<uint32_t>(t) & omask) << (l * OB);
+        else
+          w += static_cast<uint32_t>(t) << (l * OB);
+      }
+      h[j] = OS ? w : w - bias_sum;
+    }
+    if (!row_valid) continue;
+    uint32_t *dst = row32 + col / LH;
+    if (cnt < 32) {  // the last group of a channel count that is not a multiple of 32
+#pragma unroll
+      for (int j = 0; j < NH; ++j) {
+        const int c0 = j * LH;  // first channel of half-word j
+        if (c0 < cnt) {
+          const int nl = cnt - c0 < LH ? cnt - c0 : LH;
+          dst[j] = nl == LH ? h[j] : (h[j] & ((1u << (nl * OB)) - 1));
+        }
+      }
+    } else if constexpr (NH % 4 == 0) {
+      if ((reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+#pragma unroll
+        for (int v = 0; v < NH / 4; ++v)
+          reinterpret_cast<uint4 *>(dst)[v] = make_uint4(h[4 * v], h[4 * v + 1], h[4 * v + 2], h[4 * v + 3]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < NH; ++j) dst[j] = h[j];
+      }
+    } else if constexpr (NH == 2) {
+      if ((reinterpret_cast<uintptr_t>(dst) & 7) == 0)
+        *reinterpret_cast<uint2 *>(dst) = make_uint2(h[0], h[1]);
+      else
+        dst[0] = h[0], dst[1] = h[1];
+    } else {
+      dst[0] = h[0];
+    }
+  }
+}
+
+// Every other case, 16 columns at a time: split digits (acc = 16 hi + lo),
+// int32 outputs, accumulators too large for the fma path.
+template <typename WO>
+__device__ __forceinline__ void epilogue_row_general(const ConvArgs &args, uint32_t taddr, bool row_valid,
+                                                     long long m, int nb) {
   const int ch0 = nb * args.NBc;
   const int nvalid = args.K - ch0 < args.NBc ? args.K - ch0 : args.NBc;
   const bool vec_ok = (args.K % 4 == 0) && (ch0 % 4 == 0);
   const int lo = lane_lo(args.out_bits, args.out_signed), hi = lane_hi(args.out_bits, args.out_signed);
   const uint32_t omask = (1u << args.out_bits) - 1;
-  const bool bytes_path = args.packed_out && !args.out_fast;
-  volatile int *status = args.status;
-  auto wait_lane0 = [&](uint32_t bar, uint32_t parity) {
-    bool w_ok = true;
-    if (lane == 0) w_ok = ptx::mbar_wait_bounded(bar, parity, status, kWaitLimitNs);
-    return __shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0) != 0;
-  };
-  if (bytes_path && half == 1 && i >= 1 && !wait_lane0(ebar_free, static_cast<uint32_t>((i - 1) & 1))) return false;
-  // A row holds whole 32-channel groups plus 4 bytes: an odd number of 32-bit
-  // words, so the warp's 4-byte stores fall in distinct banks.
-  const int ebytes = (args.n_mma + 31) / 32 * 32 + 4;
-  uint8_t *erow = ebuf + row * ebytes;
-  for (int col = 32 * half; col < nvalid; col += 64) {
-    uint32_t r[32];
-    int v[32];
-    ptx::tmem_ld_32x32b_x32(taddr + col, r);
+  const int L = args.out_L, lw = args.out_lane_w;
+  RowPacker<WO> pk;
+  pk.dst = static_cast<WO *>(args.packed_out) + (m * args.out_wpr + ch0 / (L > 0 ? L : 1));
+  for (int col = 0; col < nvalid; col += 16) {
+    uint32_t r[16];
+    int v[16];
+    ptx::tmem_ld_32x32b_x16(taddr + col, r);
     if (args.split) {  // acc = 16 * hi + lo
-      uint32_t r2[32];
-      ptx::tmem_ld_32x32b_x32(taddr + args.n_mma + col, r2);
+      uint32_t r2[16];
+      ptx::tmem_ld_32x32b_x16(taddr + args.n_mma + col, r2);
       ptx::tmem_wait_ld();
 #pragma unroll
-      for (int k = 0; k < 32; ++k)
+      for (int k = 0; k < 16; ++k)
         v[k] = 16 * __float2int_rn(__uint_as_float(r[k])) + __float2int_rn(__uint_as_float(r2[k]));
     } else {
       ptx::tmem_wait_ld();
+      if (args.fast_acc) {  // |acc| < 2^22: the exact integer from the float's encoding
 #pragma unroll
-      for (int k = 0; k < 32; ++k) v[k] = __float2int_rn(__uint_as_float(r[k]));
+        for (int k = 0; k < 16; ++k) v[k] = floor_scaled_biased(__uint_as_float(r[k]), 1.0f) - kMagicBits;
+      } else {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) v[k] = __float2int_rn(__uint_as_float(r[k]));
+      }
     }
     if (!row_valid) continue;
-    const int cnt = nvalid - col < 32 ? nvalid - col : 32;
+    const int cnt = nvalid - col < 16 ? nvalid - col : 16;
     if (args.acc_out) {
       int32_t *dst = args.acc_out + m * args.K + ch0 + col;
-      if (cnt == 32 && vec_ok) {
+      if (cnt == 16 && vec_ok) {
 #pragma unroll
-        for (int k = 0; k < 8; ++k)
+        for (int k = 0; k < 4; ++k)
           reinterpret_cast<int4 *>(dst)[k] = make_int4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
       } else {
 #pragma unroll
-        for (int k = 0; k < 32; ++k)
+        for (int k = 0; k < 16; ++k)
           if (k < cnt) dst[k] = v[k];
       }
     }
     if (args.packed_out) {
-      uint32_t y[32];
 #pragma unroll
-      for (int k = 0; k < 32; ++k)
-        y[k] = k < cnt ? static_cast<uint32_t>(clamp_int(v[k] >> args.shift, lo, hi)) & omask : 0u;
-      if (args.out_fast) {
-        const long long w0 = m * args.out_wpr + (ch0 + col) / args.out_L;
-        const int lw = args.out_lane_w;
-        if (args.out_word64) {
-          uint64_t *dst = static_cast<uint64_t *>(args.packed_out) + w0;
-          switch (args.out_fast) {
-            case 8: pack_regs<8>(y, lw, cnt, dst); break;
-            case 16: pack_regs<16>(y, lw, cnt, dst); break;
-            default: pack_regs<32>(y, lw, cnt, dst); break;
-          }
-        } else {
-          uint32_t *dst = static_cast<uint32_t *>(args.packed_out) + w0;
-          switch (args.out_fast) {
-            case 4: pack_regs<4>(y, lw, cnt, dst); break;
-            case 8: pack_regs<8>(y, lw, cnt, dst); break;
-            case 16: pack_regs<16>(y, lw, cnt, dst); break;
-            default: pack_regs<32>(y, lw, cnt, dst); break;
-          }
-        }
-      } else {
-#pragma unroll
-        for (int k4 = 0; k4 < 8; ++k4)
-          *reinterpret_cast<uint32_t *>(erow + col + 4 * k4) =
-              y[4 * k4] | (y[4 * k4 + 1] << 8) | (y[4 * k4 + 2] << 16) | (y[4 * k4 + 3] << 24);
-      }
+      for (int k = 0; k < 16; ++k)
+        if (k < cnt) pk.put(static_cast<uint32_t>(clamp_int(v[k] >> args.shift, lo, hi)) & omask, L, lw);
     }
   }
-  if (!bytes_path) return true;
-  if (half == 1) {
-    __syncwarp();
-    if (lane == 0) ptx::mbar_arrive(ebar_full);  // this tile's bytes of the other half are written
-    return true;
-  }
-  if (!wait_lane0(ebar_full, static_cast<uint32_t>(i & 1))) return false;
-  // each output word packs L consecutive channels of this row
-  if (row_valid) {
-    const int Lo = args.out_L, lw = args.out_lane_w;
-    const int nwords = (nvalid + Lo - 1) / Lo;
-    const long long w0 = m * args.out_wpr + ch0 / Lo;
-    if (args.out_word64) {
-      uint64_t *dst = static_cast<uint64_t *>(args.packed_out) + w0;
-      for (int j = 0; j < nwords; ++j) {
-        const int c0 = j * Lo, cn = nvalid - c0 < Lo ? nvalid - c0 : Lo;
-        uint64_t wv = 0;
-        for (int l = 0; l < cn; ++l) wv |= static_cast<uint64_t>(erow[c0 + l]) << (l * lw);
-        dst[j] = wv;
-      }
-    } else {
-      uint32_t *dst = static_cast<uint32_t *>(args.packed_out) + w0;
-      for (int j = 0; j < nwords; ++j) {
-        const int c0 = j * Lo, cn = nvalid - c0 < Lo ? nvalid - c0 : Lo;
-        uint32_t wv = 0;
-        for (int l = 0; l < cn; ++l) wv |= static_cast<uint32_t>(erow[c0 + l]) << (l * lw);
-        dst[j] = wv;
-      }
+  if (args.packed_out && row_valid) pk.flush();
+}
+
+__device__ __forceinline__ void epilogue_row(const ConvArgs &args, uint32_t taddr, bool row_valid, long long m,
+                                             int nb) {
+  const bool fast = args.packed_out && !args.acc_out && !args.split && args.fast_req;
+  if (fast && args.out_lane_w == args.out_bits && (args.out_bits & (args.out_bits - 1)) == 0) {
+    switch (args.out_bits * 2 + (args.out_signed ? 1 : 0)) {
+      case 2: epilogue_row_spec<1, false>(args, taddr, row_valid, m, nb); return;
+      case 3: epilogue_row_spec<1, true>(args, taddr, row_valid, m, nb); return;
+      case 4: epilogue_row_spec<2, false>(args, taddr, row_valid, m, nb); return;
+      case 5: epilogue_row_spec<2, true>(args, taddr, row_valid, m, nb); return;
+      case 8: epilogue_row_spec<4, false>(args, taddr, row_valid, m, nb); return;
+      case 9: epilogue_row_spec<4, true>(args, taddr, row_valid, m, nb); return;
+      case 16: epilogue_row_spec<8, false>(args, taddr, row_valid, m, nb); return;
+      case 17: epilogue_row_spec<8, true>(args, taddr, row_valid, m, nb); return;
+      default: break;
     }
   }
-  __syncwarp();
-  if (lane == 0) ptx::mbar_arrive(ebar_free);  // the bytes may be overwritten
-  return true;
+  if (args.out_word64) {
+    if (fast)
+      epilogue_row_fast<uint64_t>(args, taddr, row_valid, m, nb);
+    else
+      epilogue_row_general<uint64_t>(args, taddr, row_valid, m, nb);
+  } else {
+    if (fast)
+      epilogue_row_fast<uint32_t>(args, taddr, row_valid, m, nb);
+    else
+      epilogue_row_general<uint32_t>(args, taddr, row_valid, m, nb);
+  }
 }
 
 // Issues `ksteps` (1..4) MMAs of one operand row as straight-line code.
@@ -550,10 +760,10 @@ __device__ __forceinline__ void issue_taps(uint32_t d, uint64_t a, uint64_t b, u
 //               items; each thread gathers its pixel's packed words (implicit
 //               im2col, zero padding) through a cp.async ring and widens them
 //               into a ring of A tiles.
-//   warps 10-17 epilogue: tcgen05.ld, exact int32, optional int32 store,
-//               optional requantize-and-pack; warp w reads TMEM lanes of
-//               quadrant w % 4, the two warps of a quadrant take alternate
-//               32-column groups.
+//   warps 10-17 epilogue: tcgen05.ld, exact integers, optional int32 store,
+//               optional requantize-and-pack. Warps 10-13 drain accumulator 0
+//               (the CTA's even tiles), warps 14-17 accumulator 1; warp w
+//               reads the TMEM lanes of quadrant w % 4.
 // Every wait is bounded; a role that gives up records SAMD_ETIMEOUT and stops.
 template <typename W, int BITS, bool SIGNED, bool HALO, bool FP8>
 __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant__ CUtensorMap tmap_b,
@@ -572,12 +782,10 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
   uint8_t *sOp = smem;  // HALO: 2 halo buffers; GATHER: stages_a A tiles
   uint8_t *sB = smem + args.off_b;
   uint8_t *sG = smem + args.off_g;  // packed staging
-  uint8_t *sE = smem + args.off_e;  // epilogue byte rows
   uint64_t *bars = reinterpret_cast<uint64_t *>(smem + args.off_bar);
   // barriers: full_b[STB] empty_b[STB] opfull[NO] opempty[NO] accfull[2] accempty[2] drain
-  //           ebar_full[4] ebar_free[4] (epilogue byte rows, per row quadrant)
   const int NO = HALO ? 2 : args.stages_a;
-  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 2 * STB + 2 * NO + 13);
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 2 * STB + 2 * NO + 5);
   auto full_b = [&](int s) { return ptx::smem_addr(bars + s); };
   auto empty_b = [&](int s) { return ptx::smem_addr(bars + STB + s); };
   auto opfull = [&](int s) { return ptx::smem_addr(bars + 2 * STB + s); };
@@ -585,8 +793,6 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
   auto accfull = [&](int a) { return ptx::smem_addr(bars + 2 * STB + 2 * NO + a); };
   auto accempty = [&](int a) { return ptx::smem_addr(bars + 2 * STB + 2 * NO + 2 + a); };
   const uint32_t drain_bar = ptx::smem_addr(bars + 2 * STB + 2 * NO + 4);
-  auto ebar_full = [&](int q) { return ptx::smem_addr(bars + 2 * STB + 2 * NO + 5 + q); };
-  auto ebar_free = [&](int q) { return ptx::smem_addr(bars + 2 * STB + 2 * NO + 9 + q); };
 
   volatile int *status = args.status;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -608,13 +814,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     }
     for (int a = 0; a < 2; ++a) {
       ptx::mbar_init(accfull(a), 1);
-      ptx::mbar_init(accempty(a), kEpiWarps);
+      ptx::mbar_init(accempty(a), kEpiWarps / 2);  // the warp set that drains accumulator a
     }
     ptx::mbar_init(drain_bar, 1);
-    for (int q = 0; q < 4; ++q) {
-      ptx::mbar_init(ebar_full(q), 1);
-      ptx::mbar_init(ebar_free(q), 1);
-    }
     ptx::fence_barrier_init();
   }
   ptx::tc_fence_before();
@@ -916,14 +1118,15 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     }
   } else {
     // ---- epilogue ----
+    // warp set `set` drains accumulator `set`, i.e. the CTA's tiles i with
+    // i % 2 == set; warp w reads the TMEM lanes (tile rows) of quadrant w % 4
     const int quad = warp & 3;
-    const int half = (warp - kFirstEpiWarp) / 4;
+    const int set = (warp - kFirstEpiWarp) / 4;
     const int row = quad * 32 + lane;
-    long long i = 0;
-    for (long long tile = first_tile; tile < total_tiles; tile += tile_step, ++i) {
-      const int a = static_cast<int>(i & 1);
+    long long i = set;
+    for (long long tile = first_tile + set * tile_step; tile < total_tiles; tile += 2 * tile_step, i += 2) {
       bool w_ok = true;
-      if (lane == 0) w_ok = ptx::mbar_wait_bounded(accfull(a), static_cast<uint32_t>((i >> 1) & 1), status, kWaitLimitNs);
+      if (lane == 0) w_ok = ptx::mbar_wait_bounded(accfull(set), static_cast<uint32_t>((i >> 1) & 1), status, kWaitLimitNs);
       if (!__shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0)) {
         ok = false;
         break;
@@ -947,14 +1150,11 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         m = static_cast<long long>(mt) * BM + row;
         valid = m < args.M;
       }
-      const uint32_t taddr = tmem_base + static_cast<uint32_t>(a * args.mma_n) + (static_cast<uint32_t>(quad * 32) << 16);
-      if (!epilogue_row(args, taddr, valid, m, nb, sE, row, half, ebar_full(quad), ebar_free(quad), i)) {
-        ok = false;
-        break;
-      }
+      const uint32_t taddr = tmem_base + static_cast<uint32_t>(set * args.mma_n) + (static_cast<uint32_t>(quad * 32) << 16);
+      epilogue_row(args, taddr, valid, m, nb);
       ptx::tc_fence_before();
       __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(accempty(a));
+      if (lane == 0) ptx::mbar_arrive(accempty(set));
     }
   }
 

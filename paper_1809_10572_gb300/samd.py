@@ -43,7 +43,7 @@ SAMD_NCHW, SAMD_NHWC = 0, 1
 OPS = {"add": SAMD_ADD, "sub": SAMD_SUB, "mul": SAMD_MUL, "relu": SAMD_RELU, "requant": SAMD_REQUANT}
 
 EXPORTED = ["samd_lanes_per_word", "samd_packed_words", "samd_pack", "samd_unpack", "samd_elementwise",
-            "samd_conv2d", "samd_conv2d_workspace_size", "samd_conv2d_prepare", "samd_conv2d_prepared",
+            "samd_conv2d", "samd_conv2d_workspace_size", "samd_conv2d_operand_bits", "samd_conv2d_prepare", "samd_conv2d_prepared",
             "samd_conv2d_noalloc",
             "samd_maxpool2x2", "samd_device_status", "samd_status_str", "samd_version"]
 FMT_NONE = (0, 0, 0, 0)
@@ -93,6 +93,8 @@ def load(build_if_missing: bool = True):
     lib.samd_conv2d_prepared.restype = i32
     lib.samd_conv2d_workspace_size.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, samd_fmt]
     lib.samd_conv2d_workspace_size.restype = sz
+    lib.samd_conv2d_operand_bits.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, samd_fmt]
+    lib.samd_conv2d_operand_bits.restype = i32
     lib.samd_maxpool2x2.argtypes = [samd_fmt, vp, vp, i32, i32, i32, i32, i32, vp]
     lib.samd_maxpool2x2.restype = i32
     lib.samd_device_status.argtypes, lib.samd_device_status.restype = [c.POINTER(c.c_int), i32, vp], i32
@@ -166,6 +168,11 @@ def samd_elementwise(op, fa, a, b, fo, out, n, shift=0, saturate=0, stream=None)
 
 def samd_conv2d_workspace_size(desc: samd_conv_desc, fa: samd_fmt, fw: samd_fmt) -> int:
     return int(load().samd_conv2d_workspace_size(ctypes.byref(desc), fa, fw))
+
+
+def samd_conv2d_operand_bits(desc: samd_conv_desc, fa: samd_fmt, fw: samd_fmt) -> int:
+    """8 (e4m3) or 16 (fp16): the tensor-core operand type of this convolution; 0 if rejected."""
+    return int(load().samd_conv2d_operand_bits(ctypes.byref(desc), fa, fw))
 
 
 def samd_conv2d(desc, fa, act, fw, wt, acc_out, fo, packed_out, shift, workspace, workspace_bytes=None,

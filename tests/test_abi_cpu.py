@@ -96,3 +96,25 @@ def test_conv_argument_checks(lib):
                                     None) == samd.SAMD_EINVAL
     assert samd.samd_conv2d_workspace_size(d, fa, fw) > 0
     assert samd.samd_conv2d_workspace_size(samd.ConvShape(1, 0, 8, 8, 16).desc(), fa, fw) == 0
+
+
+def test_conv_operand_type_query(lib):
+    """e4m3 holds every integer of [-16, 16] exactly (sign, 4 exponent bits,
+    3 mantissa bits: 16 = 1.000b x 2^4, 15 = 1.111b x 2^3), so lanes with
+    max|a|, max|w| <= 16 are contracted on e4m3 operands; every other format
+    (and every split-digit layer) on fp16."""
+    d = samd.ConvShape(2, 64, 16, 16, 64).desc()
+    bits = lambda ba, sa, bw, sw, desc=d: samd.samd_conv2d_operand_bits(desc, samd.fmt(ba, sa), samd.fmt(bw, sw))
+    for b in (1, 2, 3, 4):
+        for sa in (False, True):
+            for sw in (False, True):
+                assert bits(b, sa, b, sw) == 8
+    assert bits(5, True, 5, True) == 8      # [-16, 15]
+    assert bits(5, False, 4, True) == 16    # 31 > 16
+    assert bits(4, False, 5, False) == 16
+    assert bits(6, False, 2, True) == 16
+    assert bits(8, False, 8, True) == 16    # split digits
+    assert bits(8, False, 8, True, samd.ConvShape(1, 512, 8, 8, 16).desc()) == 0  # SAMD_EUNSUP
+    assert samd.samd_conv2d_operand_bits(d, samd.fmt(4, False, spacer=1), samd.fmt(4, True)) == 0
+    assert samd.samd_conv2d_operand_bits(samd.ConvShape(1, 0, 8, 8, 16).desc(), samd.fmt(4, False),
+                                         samd.fmt(4, True)) == 0
