@@ -1,7 +1,8 @@
 """Build libsamd.so in-tree for sm_103a.
 
 Each .cu translation unit under csrc/ is compiled in parallel with nvcc
-(-gencode arch=compute_103a,code=sm_103a) and the objects are linked into
+(-gencode arch=compute_103a,code=sm_103a) -- conv_inst.cu once per kernel
+instantiation group -- and the objects are linked into
 paper_1809_10572_gb300/lib/libsamd.so. A rebuild happens only when a source
 or header is newer than the library.
 """
@@ -31,8 +32,24 @@ def nvcc() -> str:
     raise RuntimeError("nvcc not found")
 
 
+INST_SRC = os.path.join(CSRC, "conv_inst.cu")
+
+
 def sources() -> list[str]:
     return sorted(glob.glob(os.path.join(CSRC, "*.cu")))
+
+
+def units() -> list[tuple[str, list[str], str]]:
+    """(source, extra nvcc flags, object name) of every translation unit:
+    each .cu once, and conv_inst.cu once per (operand type, word width, lane
+    width) -- e4m3 only for lanes of up to 5 bits."""
+    out = [(src, [], os.path.basename(src) + ".o") for src in sources() if src != INST_SRC]
+    for fp8, max_bits in ((0, 8), (1, 5)):
+        for wb in (32, 64):
+            for bits in range(1, max_bits + 1):
+                defs = [f"-DSAMD_INST_FP8={fp8}", f"-DSAMD_INST_WB={wb}", f"-DSAMD_INST_BITS={bits}"]
+                out.append((INST_SRC, defs, f"conv_inst_{'f8' if fp8 else 'f16'}_w{wb}_b{bits}.o"))
+    return out
 
 
 def _inputs() -> list[str]:
@@ -53,18 +70,21 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | N
     cc = nvcc()
     flags = NVCC_FLAGS + list(extra_flags or [])
     with tempfile.TemporaryDirectory(prefix="samd_build_") as tmp:
-        def compile_one(src: str) -> str:
-            obj = os.path.join(tmp, os.path.basename(src) + ".o")
-            cmd = [cc] + ARCH + flags + ["-c", src, "-o", obj]
+        def compile_one(unit) -> str:
+            src, defs, name = unit
+            obj = os.path.join(tmp, name)
+            cmd = [cc] + ARCH + flags + defs + ["-c", src, "-o", obj]
             r = subprocess.run(cmd, capture_output=True, text=True)
             if r.returncode != 0:
-                raise RuntimeError(f"nvcc failed on {src}:\n{r.stderr}")
+                raise RuntimeError(f"nvcc failed on {name}:\n{r.stderr}")
             if verbose and r.stderr:
-                print(r.stderr)
+                print(name, r.stderr)
             return obj
 
-        with ThreadPoolExecutor(max_workers=max(1, min(len(sources()), os.cpu_count() or 4))) as ex:
-            objs = list(ex.map(compile_one, sources()))
+        # the slowest units (the kernel instantiations) first
+        todo = sorted(units(), key=lambda u: u[0] != INST_SRC)
+        with ThreadPoolExecutor(max_workers=max(1, min(len(todo), os.cpu_count() or 4))) as ex:
+            objs = list(ex.map(compile_one, todo))
         out_tmp = os.path.join(tmp, "libsamd.so")
         cmd = [cc] + ARCH + ["-shared", "-o", out_tmp] + objs
         r = subprocess.run(cmd, capture_output=True, text=True)

@@ -147,6 +147,7 @@ EncodeTiledFn encode_tiled() {
 
 struct Plan {
   int fp8;        // e4m3 operands (kind::f8f6f4); else fp16
+  int full;       // one chunk holds all of a pixel's words (AUnpack FULL)
   int row_bytes;  // operand row: 64 (e4m3) or 128 (fp16) bytes
   int wpr, words_total, La, WC, nchunks, Kpad, NBc, n_mma, mma_n, split, nblocks, stages, Ho, Wo, gather_vec;
   int halo, Hv, Wp, nck, taps;
@@ -186,8 +187,11 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
   // e4m3 holds every integer of [-16, 16] exactly
   p.fp8 = (!p.split && max_abs(fa) <= 16 && max_abs(fw) <= 16) ? 1 : 0;
   p.row_bytes = p.fp8 ? 64 : 128;
-  p.WC = BK / p.La;
   p.wpr = static_cast<int>((d->C + p.La - 1) / p.La);
+  // FULL chunking (see AUnpack): lanes per word not dividing 64, and the
+  // pixel's words hold at most 64 channels in exactly ceil(64 / L) words
+  p.full = (BK % p.La != 0 && d->C <= BK && p.wpr == (BK + p.La - 1) / p.La) ? 1 : 0;
+  p.WC = p.full ? p.wpr : BK / p.La;
   p.words_total = d->R * d->S * p.wpr;
   p.nchunks = (p.words_total + p.WC - 1) / p.WC;
   p.Kpad = p.nchunks * BK;
@@ -506,6 +510,7 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   a.seg_used = p.seg_used;
   a.row_step = p.row_step;
   a.nck = p.nck;
+  a.full = p.full;
   a.taps = p.taps;
   // the kernel's index math runs in 32 bits
   if (static_cast<long long>(d->N) * p.Hv * p.Wp + (p.nseg + 1) * static_cast<long long>(p.Wp) + kMaxHaloRows + BM >=
@@ -531,16 +536,20 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   long long ctas = (total_tiles + kMinTilesPerCta - 1) / kMinTilesPerCta;
   if (ctas > sm_count()) ctas = sm_count();
   dim3 grid(static_cast<unsigned>(ctas));
-  const bool halo = p.halo != 0;
-  cudaError_t e;
-  if (p.fp8)
-    e = (fa.word_bits == 32 ? launch_conv_f8_w32 : launch_conv_f8_w64)(fa.bits, fa.is_signed, tmap, a, halo, grid,
-                                                                        p.smem_bytes, s);
-  else if (fa.word_bits == 32)
-    e = (fa.bits <= 4 ? launch_conv_f16_w32a : launch_conv_f16_w32b)(fa.bits, fa.is_signed, tmap, a, halo, grid,
-                                                                      p.smem_bytes, s);
-  else
-    e = launch_conv_f16_w64(fa.bits, fa.is_signed, tmap, a, halo, grid, p.smem_bytes, s);
+  static const LaunchFn kF16[2][8] = {
+      {launch_conv_f16_w32_b1, launch_conv_f16_w32_b2, launch_conv_f16_w32_b3, launch_conv_f16_w32_b4,
+       launch_conv_f16_w32_b5, launch_conv_f16_w32_b6, launch_conv_f16_w32_b7, launch_conv_f16_w32_b8},
+      {launch_conv_f16_w64_b1, launch_conv_f16_w64_b2, launch_conv_f16_w64_b3, launch_conv_f16_w64_b4,
+       launch_conv_f16_w64_b5, launch_conv_f16_w64_b6, launch_conv_f16_w64_b7, launch_conv_f16_w64_b8}};
+  static const LaunchFn kF8[2][5] = {
+      {launch_conv_f8_w32_b1, launch_conv_f8_w32_b2, launch_conv_f8_w32_b3, launch_conv_f8_w32_b4,
+       launch_conv_f8_w32_b5},
+      {launch_conv_f8_w64_b1, launch_conv_f8_w64_b2, launch_conv_f8_w64_b3, launch_conv_f8_w64_b4,
+       launch_conv_f8_w64_b5}};
+  const int wi = fa.word_bits == 64 ? 1 : 0;
+  if (p.fp8 && fa.bits > 5) return SAMD_EUNSUP;  // not reached: e4m3 only for |a| <= 16
+  const LaunchFn fn = p.fp8 ? kF8[wi][fa.bits - 1] : kF16[wi][fa.bits - 1];
+  const cudaError_t e = fn(fa.is_signed != 0, tmap, a, p.halo != 0, grid, p.smem_bytes, s);
   return e == cudaSuccess ? SAMD_OK : SAMD_ECUDA;
 }
 

@@ -30,6 +30,7 @@
 #include <cuda_fp16.h>
 
 #include <cstring>
+#include <type_traits>
 #include <utility>
 
 #include "samd_internal.cuh"
@@ -168,6 +169,7 @@ struct ConvArgs {
   int Hv, Wp;
   int nseg, seg_rows, seg_used, row_step;
   int nck;   // channel chunks per pixel (ceil(wpr / WC))
+  int full;  // AUnpack FULL: one chunk holds all the pixel's words
   int taps;  // R * S
   FastDiv fd_plane, fd_wp;  // / (Hv * Wp), / Wp
   FastDiv fd_seg;           // / seg_rows
@@ -192,12 +194,17 @@ __device__ __forceinline__ uint32_t f16x2_to_e4m3x2(uint32_t h) {
 }
 
 // Widening of one 64-position row of the A operand (one pixel, one chunk).
-template <typename W, int BITS, bool SIGNED, bool FP8>
+// A chunk is WC whole words. FULL (lanes per word not dividing 64, at most
+// 64 channels in ceil(64 / L) words): one chunk holds all the pixel's words
+// and its 64 positions are channels 0..63 -- the last word's lanes past 64
+// are padding; otherwise WC = floor(64 / L) and positions past WC * L are
+// zero.
+template <typename W, int BITS, bool SIGNED, bool FP8, bool FULL = false>
 struct AUnpack {
   static constexpr int WB = WordTraits<W>::kBits;
   static constexpr int L = WB / BITS;
-  static constexpr int WC = BK / L;        // packed words per chunk
-  static constexpr int KUSED = WC * L;     // positions holding lanes; the rest are zero
+  static constexpr int WC = FULL ? (BK + L - 1) / L : BK / L;  // packed words per chunk
+  static constexpr int KUSED = FULL ? BK : WC * L;             // positions holding lanes; the rest are zero
   static constexpr uint32_t LM = (1u << BITS) - 1;
   static constexpr uint32_t OFF = SIGNED ? (1u << (BITS - 1)) : 0u;  // offset-binary zero
   static constexpr uint32_t BIAS = 0x6400u + OFF;                   // fp16 bits of 1024 + OFF
@@ -521,17 +528,19 @@ __device__ __forceinline__ void epilogue_row_fast(const ConvArgs &args, uint32_t
   if (!args.out_fast && row_valid) pk.flush();
 }
 
-// The fast epilogue for output lanes of OB = 1, 2, 4 or 8 bits without
-// spacers: the words of a 32-channel group are built 32 bits at a time
-// (a 64-bit word is its two 32-bit halves, low half first, so the bytes are
-// the same) with compile-time shifts. Unsigned lanes are summed in the
+// The fast epilogue for output lanes of OB = 1, 2, 4, 7 or 8 bits without
+// spacers (7 only in 32-bit words): the words of a 32-channel group are built
+// 32 bits at a time (for OB dividing 32 a 64-bit word is its two 32-bit
+// halves, low half first, so the bytes are the same) with compile-time
+// shifts. Unsigned lanes are summed in the
 // biased domain and the bias sum is removed once per word; signed lanes are
 // masked to their two's complement bits first.
 template <int OB, bool OS>
 __device__ __forceinline__ void epilogue_row_spec(const ConvArgs &args, uint32_t taddr, bool row_valid, long long m,
                                                   int nb) {
-  constexpr int LH = 32 / OB;  // lanes per 32-bit half-word
-  constexpr int NH = OB;       // half-words per 32-channel group
+  constexpr int LH = 32 / OB;  // lanes per 32-bit half-word (a divisor of 32: OB = 1, 2, 4, 7, 8)
+  constexpr int NH = 32 / LH;  // half-words per 32-channel group
+  static_assert(32 % LH == 0, "whole half-words per 32-channel group");
   constexpr int32_t lo = OS ? -(1 << (OB - 1)) : 0, hi = OS ? (1 << (OB - 1)) - 1 : (1 << OB) - 1;
   constexpr int32_t blo = kMagicBits + lo, bhi = kMagicBits + hi;
   constexpr uint32_t omask = (1u << OB) - 1;
@@ -598,6 +607,56 @@ __device__ __forceinline__ void epilogue_row_spec(const ConvArgs &args, uint32_t
   }
 }
 
+__host__ __device__ constexpr int gcd_c(int a, int b) { return b == 0 ? a : gcd_c(b, a % b); }
+
+// The fast epilogue for 32-bit output words whose L = 32 / OB lanes do not
+// divide 32 (OB = 3, 5, 6: L = 10, 6, 5). Word boundaries repeat every
+// lcm(32, L) channels, so one such period (G groups of 32 columns) is
+// unrolled and every lane's word and shift are compile-time. Lanes past the
+// last channel read the biased zero, so a final partial word is zero-filled.
+template <int OB, bool OS>
+__device__ __forceinline__ void epilogue_row_period(const ConvArgs &args, uint32_t taddr, bool row_valid,
+                                                    long long m, int nb) {
+  constexpr int L = 32 / OB;
+  constexpr int G = L / gcd_c(32, L);  // lcm(32, L) / 32
+  constexpr int32_t lo = OS ? -(1 << (OB - 1)) : 0, hi = OS ? (1 << (OB - 1)) - 1 : (1 << OB) - 1;
+  constexpr int32_t blo = kMagicBits + lo, bhi = kMagicBits + hi;
+  constexpr uint32_t omask = (1u << OB) - 1;  // the low bits of kMagicBits + y are those of y
+  const int ch0 = nb * args.NBc;
+  const int nvalid = args.K - ch0 < args.NBc ? args.K - ch0 : args.NBc;
+  const float scale = args.out_scale;
+  uint32_t *dst = static_cast<uint32_t *>(args.packed_out) + (m * args.out_wpr + ch0 / L);
+  for (int c0 = 0; c0 < nvalid; c0 += 32 * G) {
+    uint32_t cur = 0;
+    bool open = false;
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const int col = c0 + 32 * g;
+      if (col >= nvalid) break;
+      uint32_t r[32];
+      ptx::tmem_ld_32x32b_x32(taddr + col, r);
+      ptx::tmem_wait_ld();
+#pragma unroll
+      for (int k = 0; k < 32; ++k) {
+        const int q = 32 * g + k;  // channel within the period (compile-time after unrolling)
+        const int l = q % L;
+        int32_t t = floor_scaled_biased(__uint_as_float(r[k]), scale);
+        t = t < blo ? blo : (t > bhi ? bhi : t);
+        if (col + k >= nvalid) t = kMagicBits;
+        cur |= (static_cast<uint32_t>(t) & omask) << (l * OB);
+        open = true;
+        if (l == L - 1) {
+          if (row_valid) *dst = cur;
+          ++dst;
+          cur = 0;
+          open = false;
+        }
+      }
+    }
+    if (open && row_valid) *dst = cur;  // the row's last, partial word
+  }
+}
+
 // Every other case, 16 columns at a time: split digits (acc = 16 hi + lo),
 // int32 outputs, accumulators too large for the fma path.
 template <typename WO>
@@ -658,14 +717,22 @@ __device__ __forceinline__ void epilogue_row_general(const ConvArgs &args, uint3
 __device__ __forceinline__ void epilogue_row(const ConvArgs &args, uint32_t taddr, bool row_valid, long long m,
                                              int nb) {
   const bool fast = args.packed_out && !args.acc_out && !args.split && args.fast_req;
-  if (fast && args.out_lane_w == args.out_bits && (args.out_bits & (args.out_bits - 1)) == 0) {
+  if (fast && args.out_lane_w == args.out_bits && (!args.out_word64 || (args.out_bits & (args.out_bits - 1)) == 0)) {
     switch (args.out_bits * 2 + (args.out_signed ? 1 : 0)) {
       case 2: epilogue_row_spec<1, false>(args, taddr, row_valid, m, nb); return;
       case 3: epilogue_row_spec<1, true>(args, taddr, row_valid, m, nb); return;
       case 4: epilogue_row_spec<2, false>(args, taddr, row_valid, m, nb); return;
       case 5: epilogue_row_spec<2, true>(args, taddr, row_valid, m, nb); return;
+      case 6: epilogue_row_period<3, false>(args, taddr, row_valid, m, nb); return;
+      case 7: epilogue_row_period<3, true>(args, taddr, row_valid, m, nb); return;
       case 8: epilogue_row_spec<4, false>(args, taddr, row_valid, m, nb); return;
       case 9: epilogue_row_spec<4, true>(args, taddr, row_valid, m, nb); return;
+      case 10: epilogue_row_period<5, false>(args, taddr, row_valid, m, nb); return;
+      case 11: epilogue_row_period<5, true>(args, taddr, row_valid, m, nb); return;
+      case 12: epilogue_row_period<6, false>(args, taddr, row_valid, m, nb); return;
+      case 13: epilogue_row_period<6, true>(args, taddr, row_valid, m, nb); return;
+      case 14: epilogue_row_spec<7, false>(args, taddr, row_valid, m, nb); return;
+      case 15: epilogue_row_spec<7, true>(args, taddr, row_valid, m, nb); return;
       case 16: epilogue_row_spec<8, false>(args, taddr, row_valid, m, nb); return;
       case 17: epilogue_row_spec<8, true>(args, taddr, row_valid, m, nb); return;
       default: break;
@@ -765,10 +832,10 @@ __device__ __forceinline__ void issue_taps(uint32_t d, uint64_t a, uint64_t b, u
 //               (the CTA's even tiles), warps 14-17 accumulator 1; warp w
 //               reads the TMEM lanes of quadrant w % 4.
 // Every wait is bounded; a role that gives up records SAMD_ETIMEOUT and stops.
-template <typename W, int BITS, bool SIGNED, bool HALO, bool FP8>
+template <typename W, int BITS, bool SIGNED, bool HALO, bool FP8, bool FULL>
 __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant__ CUtensorMap tmap_b,
                                                            const ConvArgs args) {
-  using U = AUnpack<W, BITS, SIGNED, FP8>;
+  using U = AUnpack<W, BITS, SIGNED, FP8, FULL>;
   using T = OpTraits<FP8>;
   constexpr int WC = U::WC;
   using St = Staging<W, WC>;
@@ -902,7 +969,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         }
         int words = (HALO ? args.wpr : args.words_total) - j * WC;
         if (words > WC) words = WC;
-        const int ksteps = (words * U::L + T::kKPerMma - 1) / T::kKPerMma;
+        int npos = words * U::L;
+        if (npos > BK) npos = BK;  // FULL: the last word's lanes past 64 are padding
+        const int ksteps = (npos + T::kKPerMma - 1) / T::kKPerMma;
         // No tcgen05 fence here: the operands arrived through the async proxy
         // (TMA, or stores fenced with fence.proxy.async before the producers'
         // arrive), which the mbarrier wait already orders.
@@ -1170,26 +1239,46 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
 // cudaFuncSetAttribute once per (kernel, device); defined in conv2d.cu.
 cudaError_t ensure_smem_attr(const void *kern, size_t smem);
 
+// FULL variants exist only for lane counts that do not divide 64.
+__host__ __device__ constexpr bool needs_full(int word_bits, int bits) { return 64 % (word_bits / bits) != 0; }
+
 template <typename W, int BITS, bool SIGNED, bool FP8>
 cudaError_t launch_conv(const CUtensorMap &tmap, const ConvArgs &args, bool halo, dim3 grid, size_t smem,
                         cudaStream_t s) {
-  auto kern = halo ? conv_kernel<W, BITS, SIGNED, true, FP8> : conv_kernel<W, BITS, SIGNED, false, FP8>;
+  constexpr bool kHasFull = needs_full(WordTraits<W>::kBits, BITS);
+  auto kern = halo ? conv_kernel<W, BITS, SIGNED, true, FP8, false> : conv_kernel<W, BITS, SIGNED, false, FP8, false>;
+  if constexpr (kHasFull) {
+    if (args.full)
+      kern = halo ? conv_kernel<W, BITS, SIGNED, true, FP8, true> : conv_kernel<W, BITS, SIGNED, false, FP8, true>;
+  }
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void *>(kern), smem);
   if (e != cudaSuccess) return e;
   kern<<<grid, kThreads, smem, s>>>(tmap, args);
   return cudaGetLastError();
 }
 
-// Launchers by operand type, word width and lane width (one translation unit
-// each, so that they compile in parallel).
-#define SAMD_CONV_LAUNCHER(name)                                                                             \
-  cudaError_t name(int bits, bool is_signed, const CUtensorMap &tmap, const ConvArgs &args, bool halo, dim3 grid, \
-                   size_t smem, cudaStream_t s);
-SAMD_CONV_LAUNCHER(launch_conv_f16_w32a)  // 1-4-bit lanes
-SAMD_CONV_LAUNCHER(launch_conv_f16_w32b)  // 5-8-bit lanes
-SAMD_CONV_LAUNCHER(launch_conv_f16_w64)
-SAMD_CONV_LAUNCHER(launch_conv_f8_w32)
-SAMD_CONV_LAUNCHER(launch_conv_f8_w64)
+// Launchers, one per (operand type, activation word width, lane width), each
+// compiled from conv_inst.cu in its own unit.
+using LaunchFn = cudaError_t (*)(bool is_signed, const CUtensorMap &tmap, const ConvArgs &args, bool halo, dim3 grid,
+                                 size_t smem, cudaStream_t s);
+#define SAMD_CONV_LAUNCHER(name) \
+  cudaError_t name(bool is_signed, const CUtensorMap &tmap, const ConvArgs &args, bool halo, dim3 grid, size_t smem, \
+                   cudaStream_t s);
+#define SAMD_CONV_LAUNCHERS(t, wb)                                                                          \
+  SAMD_CONV_LAUNCHER(launch_conv_##t##_w##wb##_b1) SAMD_CONV_LAUNCHER(launch_conv_##t##_w##wb##_b2)        \
+  SAMD_CONV_LAUNCHER(launch_conv_##t##_w##wb##_b3) SAMD_CONV_LAUNCHER(launch_conv_##t##_w##wb##_b4)        \
+  SAMD_CONV_LAUNCHER(launch_conv_##t##_w##wb##_b5)
+SAMD_CONV_LAUNCHERS(f16, 32)
+SAMD_CONV_LAUNCHERS(f16, 64)
+SAMD_CONV_LAUNCHERS(f8, 32)
+SAMD_CONV_LAUNCHERS(f8, 64)
+SAMD_CONV_LAUNCHER(launch_conv_f16_w32_b6)
+SAMD_CONV_LAUNCHER(launch_conv_f16_w32_b7)
+SAMD_CONV_LAUNCHER(launch_conv_f16_w32_b8)
+SAMD_CONV_LAUNCHER(launch_conv_f16_w64_b6)
+SAMD_CONV_LAUNCHER(launch_conv_f16_w64_b7)
+SAMD_CONV_LAUNCHER(launch_conv_f16_w64_b8)
+#undef SAMD_CONV_LAUNCHERS
 #undef SAMD_CONV_LAUNCHER
 
 }  // namespace conv
