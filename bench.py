@@ -213,7 +213,7 @@ def workload_config(args, layers):
     }[args.workload]
     return {"workload": desc, "layers": len(layers), "macs_per_step": workloads.total_macs(layers),
             "l2": "flushed before every step (512 MiB write, then 512 MiB read); inputs resident in HBM",
-            "weights": "prepared once into the fp16 operand layout (samd_conv2d_prepare), not in the step",
+            "weights": "prepared once into the tensor-core operand layout (samd_conv2d_prepare), not in the step",
             "launch": f"one CUDA graph per step; independent layers fanned out over {args.streams} streams",
             "parallelism": f"replicas x{args.gpus}"}
 
