@@ -148,6 +148,7 @@ EncodeTiledFn encode_tiled() {
 struct Plan {
   int fp8;        // e4m3 operands (kind::f8f6f4); else fp16
   int full;       // one chunk holds all of a pixel's words (AUnpack FULL)
+  int hv;         // tile of hv halves of 128 output positions
   int row_bytes;  // operand row: 64 (e4m3) or 128 (fp16) bytes
   int wpr, words_total, La, WC, nchunks, Kpad, NBc, n_mma, mma_n, split, nblocks, stages, Ho, Wo, gather_vec;
   int halo, Hv, Wp, nck, taps;
@@ -166,7 +167,7 @@ long long max_abs(samd_fmt f) { return f.is_signed ? (1LL << (f.bits - 1)) : ((1
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-constexpr int kMaxHaloRows = 640;
+constexpr int kMaxHaloRows = 1024;
 constexpr int kMinTilesPerCta = 4;
 
 // Tiling, reduction order, operand type and exactness mode for one
@@ -233,44 +234,57 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
     p.off_bar = static_cast<uint32_t>(round_up(p.off_e + e_bytes, 16));
     p.smem_bytes = 1024 + p.off_bar + bar_bytes(p.stages, op_stages);  // + alignment slack of the base
   };
-  p.grid_m = (p.M + BM - 1) / BM;
   p.taps = d->R * d->S;
   p.nck = (p.wpr + p.WC - 1) / p.WC;
   p.Hv = d->H + 2 * d->pad;
   p.Wp = d->W + 2 * d->pad;
-  p.halo = 0;
-  p.b_resident = 0;
-  p.stages_a = 0;
-  p.nseg = p.seg_rows = p.seg_used = p.row_step = 0;
-  // Halo mode: stride 1, several taps, little padded-grid waste, halo fits.
-  // The halo is either the contiguous run of virtual rows the tile touches,
-  // or (wide images) one segment of 128 + S - 1 rows per filter row.
-  if (d->stride == 1 && p.taps >= 2 && p.M > 0) {
-    const int contig = BM + (d->R - 1) * p.Wp + (d->S - 1);
-    const int seg_used = BM + d->S - 1, seg_rows = (seg_used + 7) / 8 * 8;
-    if (d->R * seg_rows < (contig + 7) / 8 * 8) {
-      p.nseg = d->R;
-      p.seg_rows = seg_rows;
-      p.seg_used = seg_used;
-      p.row_step = seg_rows;
-    } else {
-      p.nseg = 1;
-      p.seg_rows = (contig + 7) / 8 * 8;
-      p.seg_used = contig;
-      p.row_step = p.Wp;
-    }
-    const int halo_rows = p.nseg * p.seg_rows;
-    const double waste = static_cast<double>(d->N) * p.Hv * p.Wp / static_cast<double>(p.M);
-    const size_t halo_bytes = round_up(static_cast<size_t>(halo_rows) * p.row_bytes, 1024);
-    const size_t stage_g = round_up(static_cast<size_t>(halo_rows) * srow, 16);
-    const size_t fixed = 2 * halo_bytes + 2 * stage_g + e_bytes + 1024;
-    const int ntiles_b = p.nck * p.taps;
-    if (halo_rows <= kMaxHaloRows && waste <= 1.16 && fixed + 2 * bst + bar_bytes(2, 2) <= kBudget) {
+  const int nchunks_gather = p.nchunks;
+  // One configuration: operand mode (halo or gather) and tile halves hv.
+  // Returns false if it does not fit, or if `need_resident` and the weights
+  // would not stay resident.
+  auto place = [&](bool halo, int hv, bool need_resident) -> bool {
+    const int bmt = BM * hv;
+    p.hv = hv;
+    p.halo = 0;
+    p.b_resident = 0;
+    p.stages_a = 0;
+    p.nseg = p.seg_rows = p.seg_used = p.row_step = 0;
+    p.nchunks = nchunks_gather;
+    p.Kpad = p.nchunks * BK;
+    p.grid_m = (p.M + bmt - 1) / bmt;
+    if (halo) {
+      // Halo mode: stride 1, several taps, little padded-grid waste, halo
+      // fits. The halo is either the contiguous run of virtual rows the tile
+      // touches, or (wide images) one segment of bmt + S - 1 rows per filter
+      // row.
+      if (d->stride != 1 || p.taps < 2 || p.M == 0) return false;
+      const int contig = bmt + (d->R - 1) * p.Wp + (d->S - 1);
+      const int seg_used = bmt + d->S - 1, seg_rows = (seg_used + 7) / 8 * 8;
+      if (d->R * seg_rows < (contig + 7) / 8 * 8) {
+        p.nseg = d->R;
+        p.seg_rows = seg_rows;
+        p.seg_used = seg_used;
+        p.row_step = seg_rows;
+      } else {
+        p.nseg = 1;
+        p.seg_rows = (contig + 7) / 8 * 8;
+        p.seg_used = contig;
+        p.row_step = p.Wp;
+      }
+      const int halo_rows = p.nseg * p.seg_rows;
+      const double waste = static_cast<double>(d->N) * p.Hv * p.Wp / static_cast<double>(p.M);
+      const size_t halo_bytes = round_up(static_cast<size_t>(halo_rows) * p.row_bytes, 1024);
+      const size_t stage_g = round_up(static_cast<size_t>(halo_rows) * srow, 16);
+      const size_t fixed = 2 * halo_bytes + 2 * stage_g + e_bytes + 1024;
+      const int ntiles_b = p.nck * p.taps;
+      if (halo_rows > kMaxHaloRows || waste > 1.16 || fixed + 2 * bst + bar_bytes(2, 2) > kBudget) return false;
+      const bool res = p.nblocks == 1 && fixed + ntiles_b * bst + bar_bytes(ntiles_b, 2) <= kBudget;
+      if (need_resident && !res) return false;
       p.halo = 1;
       p.nchunks = ntiles_b;
       p.Kpad = ntiles_b * BK;
-      p.grid_m = (static_cast<long long>(d->N) * p.Hv * p.Wp + BM - 1) / BM;
-      if (p.nblocks == 1 && fixed + ntiles_b * bst + bar_bytes(ntiles_b, 2) <= kBudget) {
+      p.grid_m = (static_cast<long long>(d->N) * p.Hv * p.Wp + bmt - 1) / bmt;
+      if (res) {
         p.b_resident = 1;
         p.stages = ntiles_b;
       } else {
@@ -280,18 +294,17 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
       p.op_stride = static_cast<uint32_t>(halo_bytes);
       p.g_stride = static_cast<uint32_t>(stage_g);
       finish(2 * halo_bytes, 2 * stage_g, 2);
-    } else {
-      p.nseg = p.seg_rows = p.seg_used = p.row_step = 0;
+      return true;
     }
-  }
-  if (!p.halo) {
-    const size_t tile_bytes = static_cast<size_t>(BM) * p.row_bytes;
+    const size_t tile_bytes = static_cast<size_t>(bmt) * p.row_bytes;
     const size_t group_slots = static_cast<size_t>(kGatherDepth) * BM * srow;  // one producer group's ring
     for (int sta = 4; sta >= 2; --sta) {
       const size_t fixed = sta * tile_bytes + 2 * group_slots + e_bytes + 1024;
       if (fixed + 2 * bst + bar_bytes(2, sta) > kBudget) continue;
+      const bool res = p.nblocks == 1 && fixed + p.nchunks * bst + bar_bytes(p.nchunks, sta) <= kBudget;
+      if (need_resident && !res) continue;
       p.stages_a = sta;
-      if (p.nblocks == 1 && fixed + p.nchunks * bst + bar_bytes(p.nchunks, sta) <= kBudget) {
+      if (res) {
         p.b_resident = 1;
         p.stages = p.nchunks;
       } else {
@@ -301,12 +314,24 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
       p.op_stride = static_cast<uint32_t>(tile_bytes);
       p.g_stride = static_cast<uint32_t>(group_slots);
       finish(sta * tile_bytes, 2 * group_slots, sta);
-      break;
+      return true;
     }
-    if (p.stages_a == 0) return SAMD_EUNSUP;  // operand tiles do not fit (not reached for N <= 256)
-  }
+    return false;
+  };
+  // Preference: resident weights, then halo over gather, then two-half tiles
+  // (two accumulators of 2 * mma_n TMEM columns each: mma_n <= 128).
+  const bool two = p.mma_n <= 128;
+  bool placed = false;
+  for (int need_res = (p.nblocks == 1 ? 1 : 0); need_res >= 0 && !placed; --need_res)
+    for (int mode = 0; mode < 4 && !placed; ++mode) {
+      const bool halo = mode < 2;
+      const int hv = (mode % 2 == 0) ? 2 : 1;
+      if (hv == 2 && !two) continue;
+      placed = place(halo, hv, need_res != 0);
+    }
+  if (!placed) return SAMD_EUNSUP;  // operand tiles do not fit (not reached for N <= 256)
   uint32_t cols = 32;
-  while (cols < static_cast<uint32_t>(2 * p.mma_n)) cols <<= 1;  // two accumulators
+  while (cols < static_cast<uint32_t>(2 * p.hv * p.mma_n)) cols <<= 1;  // two accumulators of hv halves
   p.tmem_cols = cols;
   p.ws_bytes = static_cast<size_t>(p.nblocks) * p.mma_n * p.Kpad * (p.fp8 ? 1 : 2);
   return SAMD_OK;
@@ -323,7 +348,8 @@ bool layout_ok(const Plan &p) {
   return p.stages >= 1 && NO >= 2 && op_bytes <= p.off_b &&
          p.off_b + static_cast<size_t>(p.stages) * p.b_bytes <= p.off_g && p.off_g + 2 * p.g_stride <= p.off_e &&
          p.off_e <= p.off_bar && 1023 + p.off_bar + bars <= p.smem_bytes && p.op_stride % 1024 == 0 &&
-         p.off_b % 1024 == 0 && p.b_bytes % 1024 == 0 && p.off_bar % 8 == 0 && 2 * p.mma_n <= 512;
+         p.off_b % 1024 == 0 && p.b_bytes % 1024 == 0 && p.off_bar % 8 == 0 && 2 * p.hv * p.mma_n <= 512 &&
+         (p.hv == 1 || p.hv == 2);
 }
 
 // Device address of a __device__ symbol on the current device, looked up
@@ -511,9 +537,10 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   a.row_step = p.row_step;
   a.nck = p.nck;
   a.full = p.full;
+  a.hv = p.hv;
   a.taps = p.taps;
   // the kernel's index math runs in 32 bits
-  if (static_cast<long long>(d->N) * p.Hv * p.Wp + (p.nseg + 1) * static_cast<long long>(p.Wp) + kMaxHaloRows + BM >=
+  if (static_cast<long long>(d->N) * p.Hv * p.Wp + (p.nseg + 1) * static_cast<long long>(p.Wp) + kMaxHaloRows + 2 * BM >=
           (1LL << 31) ||
       p.M >= (1LL << 31) || p.grid_m * p.nblocks >= (1LL << 31))
     return SAMD_EUNSUP;
@@ -533,7 +560,8 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   // a small layer keeps at least kMinTilesPerCta tiles per CTA, leaving SMs
   // to independent layers issued on other streams
   const long long total_tiles = p.grid_m * p.nblocks;
-  long long ctas = (total_tiles + kMinTilesPerCta - 1) / kMinTilesPerCta;
+  const int min_tiles = kMinTilesPerCta / p.hv;  // at least 512 output positions per CTA
+  long long ctas = (total_tiles + min_tiles - 1) / min_tiles;
   if (ctas > sm_count()) ctas = sm_count();
   dim3 grid(static_cast<unsigned>(ctas));
   static const LaunchFn kF16[2][8] = {

@@ -170,6 +170,7 @@ struct ConvArgs {
   int nseg, seg_rows, seg_used, row_step;
   int nck;   // channel chunks per pixel (ceil(wpr / WC))
   int full;  // AUnpack FULL: one chunk holds all the pixel's words
+  int hv;    // tile of hv halves of 128 output positions (1 or 2)
   int taps;  // R * S
   FastDiv fd_plane, fd_wp;  // / (Hv * Wp), / Wp
   FastDiv fd_seg;           // / seg_rows
@@ -760,27 +761,36 @@ __device__ __forceinline__ void mma_op(uint32_t d, uint64_t a, uint64_t b, uint3
     ptx::mma_f16(d, a, b, idesc, acc);
 }
 
-template <bool FP8>
-__device__ __forceinline__ void mma_ksteps(int ksteps, uint32_t d, uint64_t a, uint64_t b, uint32_t idesc,
-                                           uint32_t acc) {
+// For a tile of HV halves of 128 rows, each k-step issues one MMA per half:
+// half h accumulates into d + h * dn from A rows 128 h on (a + h * ah).
+template <bool FP8, int HV>
+__device__ __forceinline__ void mma_kstep(uint32_t d, uint32_t dn, uint64_t a, uint64_t ah, uint64_t b, uint32_t idesc,
+                                          uint32_t acc) {
+  mma_op<FP8>(d, a, b, idesc, acc);
+  if constexpr (HV == 2) mma_op<FP8>(d + dn, a + ah, b, idesc, acc);
+}
+
+template <bool FP8, int HV>
+__device__ __forceinline__ void mma_ksteps(int ksteps, uint32_t d, uint32_t dn, uint64_t a, uint64_t ah, uint64_t b,
+                                           uint32_t idesc, uint32_t acc) {
   switch (ksteps) {
     case 4:
-      mma_op<FP8>(d, a, b, idesc, acc);
-      mma_op<FP8>(d, a + 2, b + 2, idesc, 1u);
-      mma_op<FP8>(d, a + 4, b + 4, idesc, 1u);
-      mma_op<FP8>(d, a + 6, b + 6, idesc, 1u);
+      mma_kstep<FP8, HV>(d, dn, a, ah, b, idesc, acc);
+      mma_kstep<FP8, HV>(d, dn, a + 2, ah, b + 2, idesc, 1u);
+      mma_kstep<FP8, HV>(d, dn, a + 4, ah, b + 4, idesc, 1u);
+      mma_kstep<FP8, HV>(d, dn, a + 6, ah, b + 6, idesc, 1u);
       break;
     case 3:
-      mma_op<FP8>(d, a, b, idesc, acc);
-      mma_op<FP8>(d, a + 2, b + 2, idesc, 1u);
-      mma_op<FP8>(d, a + 4, b + 4, idesc, 1u);
+      mma_kstep<FP8, HV>(d, dn, a, ah, b, idesc, acc);
+      mma_kstep<FP8, HV>(d, dn, a + 2, ah, b + 2, idesc, 1u);
+      mma_kstep<FP8, HV>(d, dn, a + 4, ah, b + 4, idesc, 1u);
       break;
     case 2:
-      mma_op<FP8>(d, a, b, idesc, acc);
-      mma_op<FP8>(d, a + 2, b + 2, idesc, 1u);
+      mma_kstep<FP8, HV>(d, dn, a, ah, b, idesc, acc);
+      mma_kstep<FP8, HV>(d, dn, a + 2, ah, b + 2, idesc, 1u);
       break;
     default:
-      mma_op<FP8>(d, a, b, idesc, acc);
+      mma_kstep<FP8, HV>(d, dn, a, ah, b, idesc, acc);
       break;
   }
 }
@@ -790,13 +800,13 @@ __device__ __forceinline__ void mma_ksteps(int ksteps, uint32_t d, uint64_t a, u
 // operand one row further on, skipping a_skip16 at the end of each filter
 // row (HALO); straight-line issue keeps the tensor core fed. Descriptors
 // advance in 16-byte units of their start-address field.
-template <bool FP8>
-__device__ __forceinline__ void issue_taps(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, int ksteps, int taps,
-                                           int S, uint32_t a_row16, uint32_t a_skip16, uint32_t b_step16,
-                                           uint32_t acc) {
+template <bool FP8, int HV>
+__device__ __forceinline__ void issue_taps(uint32_t d, uint32_t dn, uint64_t a, uint64_t ah, uint64_t b, uint32_t idesc,
+                                           int ksteps, int taps, int S, uint32_t a_row16, uint32_t a_skip16,
+                                           uint32_t b_step16, uint32_t acc) {
   int s = 0;
   for (int t = 0; t < taps; ++t) {
-    mma_ksteps<FP8>(ksteps, d, a, b, idesc, acc);
+    mma_ksteps<FP8, HV>(ksteps, d, dn, a, ah, b, idesc, acc);
     acc = 1;
     b += b_step16;
     a += a_row16;
@@ -810,7 +820,9 @@ __device__ __forceinline__ void issue_taps(uint32_t d, uint64_t a, uint64_t b, u
 // ---- the persistent convolution kernel ----------------------------------------
 //
 // One CTA per SM loops over output tiles (tile = blockIdx.x + i * gridDim.x;
-// tile = nb * grid_m + mt: channel block nb, 128-position tile mt). Eighteen
+// tile = nb * grid_m + mt: channel block nb, position tile mt of 128 * HV
+// positions; HV = 2 issues each k-step's MMA for both 128-row halves and
+// halves the synchronization per MMA). Eighteen
 // warps with fixed roles, connected by mbarrier rings:
 //   warp 0      TMEM allocation; lane 0 streams weight tiles with TMA. When
 //               the layer has one channel block and all its weight tiles fit,
@@ -832,10 +844,11 @@ __device__ __forceinline__ void issue_taps(uint32_t d, uint64_t a, uint64_t b, u
 //               (the CTA's even tiles), warps 14-17 accumulator 1; warp w
 //               reads the TMEM lanes of quadrant w % 4.
 // Every wait is bounded; a role that gives up records SAMD_ETIMEOUT and stops.
-template <typename W, int BITS, bool SIGNED, bool HALO, bool FP8, bool FULL>
+template <typename W, int BITS, bool SIGNED, bool HALO, bool FP8, bool FULL, int HV>
 __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant__ CUtensorMap tmap_b,
                                                            const ConvArgs args) {
   using U = AUnpack<W, BITS, SIGNED, FP8, FULL>;
+  constexpr int BMT = BM * HV;  // output positions per tile
   using T = OpTraits<FP8>;
   constexpr int WC = U::WC;
   using St = Staging<W, WC>;
@@ -876,12 +889,12 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       ptx::mbar_init(empty_b(s), 1);
     }
     for (int s = 0; s < NO; ++s) {
-      ptx::mbar_init(opfull(s), HALO ? kProdWarps : kProdWarps / 2);
+      ptx::mbar_init(opfull(s), (HALO || HV == 2) ? kProdWarps : kProdWarps / 2);
       ptx::mbar_init(opempty(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
       ptx::mbar_init(accfull(a), 1);
-      ptx::mbar_init(accempty(a), kEpiWarps / 2);  // the warp set that drains accumulator a
+      ptx::mbar_init(accempty(a), HV == 2 ? kEpiWarps : kEpiWarps / 2);  // the warps that drain accumulator a
     }
     ptx::mbar_init(drain_bar, 1);
     ptx::fence_barrier_init();
@@ -948,6 +961,8 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     const int nops = HALO ? args.nck : nchunks;  // operand stages per tile
     const int taps_here = HALO ? args.taps : 1;
     constexpr uint32_t a_row16 = T::kRowBytes / 16;  // one operand row in descriptor units
+    constexpr uint64_t a_half16 = static_cast<uint64_t>(BM) * a_row16;  // the second half's first A row
+    const uint32_t dn = static_cast<uint32_t>(args.mma_n);          // the second half's accumulator columns
     const uint32_t a_skip16 = HALO ? static_cast<uint32_t>(args.row_step - args.S) * a_row16 : 0u;
     if (resident)  // resident weights: wait for all of them once
       for (int c = 0; c < nchunks && ok; ++c)
@@ -960,7 +975,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         break;
       }
       ptx::tc_fence_after();  // the epilogue's reads of this accumulator are complete
-      const uint32_t tmem_d = tmem_base + static_cast<uint32_t>(a * args.mma_n);
+      const uint32_t tmem_d = tmem_base + static_cast<uint32_t>(a * HV * args.mma_n);
       uint32_t acc = 0;
       for (int j = 0; j < nops && ok; ++j) {
         if (!wait(opfull(so), opar)) {
@@ -979,7 +994,8 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         if (resident) {
           const uint64_t b0 = T::desc(sB_addr + (HALO ? j * taps_here : j) * b_bytes);
           if (ptx::elect_one())
-            issue_taps<FP8>(tmem_d, a0, b0, idesc, ksteps, taps_here, args.S, a_row16, a_skip16, b_bytes >> 4, acc);
+            issue_taps<FP8, HV>(tmem_d, dn, a0, a_half16, b0, idesc, ksteps, taps_here, args.S, a_row16, a_skip16,
+                                b_bytes >> 4, acc);
           __syncwarp();
           acc = 1;
         } else {
@@ -992,7 +1008,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
             }
             const uint64_t bdesc = T::desc(sB_addr + sb * b_bytes);
             if (ptx::elect_one()) {
-              mma_ksteps<FP8>(ksteps, tmem_d, adesc, bdesc, idesc, acc);
+              mma_ksteps<FP8, HV>(ksteps, tmem_d, dn, adesc, a_half16, bdesc, idesc, acc);
               ptx::mma_commit(empty_b(sb));
             }
             __syncwarp();
@@ -1049,7 +1065,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       // items k = (tile i, channel chunk j), in the MMA's order
       auto gather = [&](long long tile, int j, int slot) {
         const uint32_t mt = static_cast<uint32_t>(tile) - fdiv(static_cast<uint32_t>(tile), args.fd_gm) * args.fd_gm.d;
-        const uint32_t v0 = mt * BM;
+        const uint32_t v0 = mt * BMT;
         const uint32_t dst0 = ptx::smem_addr(sG + slot * args.g_stride);
         for (int hr = t; hr < halo_rows; hr += kProdThreads) {
           const int off = voff(hr);
@@ -1114,9 +1130,12 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       }
       ptx::cp_async_wait<0>();
     } else {
-      // GATHER: group grp (four warps) takes items grp, grp + 2, ...; thread
-      // row of the group owns row `row` of every A tile it fills
-      const int grp = t / BM, row = t % BM;
+      // GATHER: with one-half tiles group grp (four warps) takes items grp,
+      // grp + 2, ...; with two-half tiles both groups take every item, group
+      // grp filling rows 128 grp .. 128 grp + 127. A thread owns one row.
+      const int grp = t / BM;
+      const int row = (HV == 2 ? grp * BM : 0) + t % BM;  // row of the A tile
+      constexpr int kItemStep = HV == 2 ? 1 : 2;
       AGather<W, WC> g;
       g.act = act;
       g.H = args.H;
@@ -1130,7 +1149,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       auto set_tile = [&](long long tile) {
         const uint32_t tl = static_cast<uint32_t>(tile);
         const uint32_t mt = tl - fdiv(tl, args.fd_gm) * args.fd_gm.d;
-        const uint32_t m = mt * BM + row;
+        const uint32_t m = mt * BMT + row;
         g.row_valid = m < static_cast<uint64_t>(args.M);
         const uint32_t mm = g.row_valid ? m : 0u;
         const uint32_t tq = fdiv(mm, args.fd_wo);
@@ -1140,7 +1159,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         g.n = static_cast<int>(nq);
       };
       constexpr uint32_t kSlotBytes = BM * St::kRowBytes;
-      const uint32_t slot0 = ptx::smem_addr(sG) + grp * (kGatherDepth * kSlotBytes) + row * St::kRowBytes;
+      const uint32_t slot0 = ptx::smem_addr(sG) + grp * (kGatherDepth * kSlotBytes) + (t % BM) * St::kRowBytes;
       // issue side: this group's item (itile, ic), kGatherDepth ahead of the consume side
       long long itile = first_tile;
       int ic = 0;
@@ -1150,14 +1169,14 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
           itile += tile_step;
         }
       };
-      if (grp == 1) step();
+      if (HV == 1 && grp == 1) step();
       if (itile < total_tiles) set_tile(itile);
       auto issue_next = [&](int slot) {
         if (itile < total_tiles) {
           g.issue(ic, slot0 + slot * kSlotBytes);
           const long long prev = itile;
           step();
-          step();
+          if (kItemStep == 2) step();
           if (itile != prev && itile < total_tiles) set_tile(itile);
         }
         ptx::cp_async_commit();
@@ -1166,10 +1185,10 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       for (int d = 0; d < kGatherDepth; ++d) issue_next(d);
       const long long items = ((total_tiles - first_tile + tile_step - 1) / tile_step) * nchunks;
       int slot = 0;
-      for (long long k = grp; k < items; k += 2) {
+      for (long long k = HV == 2 ? 0 : grp; k < items; k += kItemStep) {
         ptx::cp_async_wait<kGatherDepth - 1>();
         W cur[WC];
-        load_staged<W, WC>(sG + grp * (kGatherDepth * kSlotBytes) + slot * kSlotBytes + row * St::kRowBytes, cur);
+        load_staged<W, WC>(sG + grp * (kGatherDepth * kSlotBytes) + slot * kSlotBytes + (t % BM) * St::kRowBytes, cur);
         const int sa = static_cast<int>(k % NO);
         const long long round = k / NO;
         if (round > 0 && !wait_lane0(opempty(sa), static_cast<uint32_t>((round - 1) & 1))) {
@@ -1187,15 +1206,19 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     }
   } else {
     // ---- epilogue ----
-    // warp set `set` drains accumulator `set`, i.e. the CTA's tiles i with
-    // i % 2 == set; warp w reads the TMEM lanes (tile rows) of quadrant w % 4
+    // One-half tiles: warp set `set` drains accumulator `set`, i.e. the CTA's
+    // tiles i with i % 2 == set. Two-half tiles: both sets drain every tile,
+    // set `set` its half `set`. Warp w reads the TMEM lanes of quadrant w % 4.
     const int quad = warp & 3;
     const int set = (warp - kFirstEpiWarp) / 4;
     const int row = quad * 32 + lane;
-    long long i = set;
-    for (long long tile = first_tile + set * tile_step; tile < total_tiles; tile += 2 * tile_step, i += 2) {
+    constexpr int kTileStep = HV == 2 ? 1 : 2;
+    long long i = HV == 2 ? 0 : set;
+    for (long long tile = first_tile + (HV == 2 ? 0 : set) * tile_step; tile < total_tiles;
+         tile += kTileStep * tile_step, i += kTileStep) {
+      const int acc_i = HV == 2 ? static_cast<int>(i & 1) : set;  // accumulator of this tile
       bool w_ok = true;
-      if (lane == 0) w_ok = ptx::mbar_wait_bounded(accfull(set), static_cast<uint32_t>((i >> 1) & 1), status, kWaitLimitNs);
+      if (lane == 0) w_ok = ptx::mbar_wait_bounded(accfull(acc_i), static_cast<uint32_t>((i >> 1) & 1), status, kWaitLimitNs);
       if (!__shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0)) {
         ok = false;
         break;
@@ -1207,8 +1230,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       const uint32_t mt = tl - nbu * args.fd_gm.d;
       bool valid;
       long long m;
+      const int trow = (HV == 2 ? set * BM : 0) + row;  // row of the tile
       if (HALO) {
-        const uint32_t v = mt * BM + row;
+        const uint32_t v = mt * BMT + trow;
         const uint32_t img = fdiv(v, args.fd_plane);
         const uint32_t rem = v - img * args.fd_plane.d;
         const uint32_t oh = fdiv(rem, args.fd_wp);
@@ -1216,14 +1240,15 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         valid = static_cast<int>(img) < args.N && static_cast<int>(oh) < args.Ho && static_cast<int>(ow) < args.Wo;
         m = (static_cast<long long>(img) * args.Ho + oh) * args.Wo + ow;
       } else {
-        m = static_cast<long long>(mt) * BM + row;
+        m = static_cast<long long>(mt) * BMT + trow;
         valid = m < args.M;
       }
-      const uint32_t taddr = tmem_base + static_cast<uint32_t>(set * args.mma_n) + (static_cast<uint32_t>(quad * 32) << 16);
+      const uint32_t taddr = tmem_base + static_cast<uint32_t>((acc_i * HV + (HV == 2 ? set : 0)) * args.mma_n) +
+                             (static_cast<uint32_t>(quad * 32) << 16);
       epilogue_row(args, taddr, valid, m, nb);
       ptx::tc_fence_before();
       __syncwarp();
-      if (lane == 0) ptx::mbar_arrive(accempty(set));
+      if (lane == 0) ptx::mbar_arrive(accempty(acc_i));
     }
   }
 
@@ -1246,10 +1271,17 @@ template <typename W, int BITS, bool SIGNED, bool FP8>
 cudaError_t launch_conv(const CUtensorMap &tmap, const ConvArgs &args, bool halo, dim3 grid, size_t smem,
                         cudaStream_t s) {
   constexpr bool kHasFull = needs_full(WordTraits<W>::kBits, BITS);
-  auto kern = halo ? conv_kernel<W, BITS, SIGNED, true, FP8, false> : conv_kernel<W, BITS, SIGNED, false, FP8, false>;
+  using K = void (*)(const CUtensorMap, const ConvArgs);
+  K kern;
+  if (args.hv == 2)
+    kern = halo ? conv_kernel<W, BITS, SIGNED, true, FP8, false, 2> : conv_kernel<W, BITS, SIGNED, false, FP8, false, 2>;
+  else
+    kern = halo ? conv_kernel<W, BITS, SIGNED, true, FP8, false, 1> : conv_kernel<W, BITS, SIGNED, false, FP8, false, 1>;
   if constexpr (kHasFull) {
-    if (args.full)
-      kern = halo ? conv_kernel<W, BITS, SIGNED, true, FP8, true> : conv_kernel<W, BITS, SIGNED, false, FP8, true>;
+    if (args.full && args.hv == 2)
+      kern = halo ? conv_kernel<W, BITS, SIGNED, true, FP8, true, 2> : conv_kernel<W, BITS, SIGNED, false, FP8, true, 2>;
+    else if (args.full)
+      kern = halo ? conv_kernel<W, BITS, SIGNED, true, FP8, true, 1> : conv_kernel<W, BITS, SIGNED, false, FP8, true, 1>;
   }
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void *>(kern), smem);
   if (e != cudaSuccess) return e;
