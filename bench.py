@@ -86,6 +86,14 @@ class Dist:
             self.dist.destroy_process_group()
 
 
+def whole_job_rate(d: Dist, units_per_step: float, steps: int, local_seconds: float):
+    """Weak scaling over replicas: every rank runs `steps` steps of
+    `units_per_step` units; the job took as long as its slowest rank. Returns
+    (units per second over all ranks, ms per step of the slowest rank)."""
+    slowest = d.max(local_seconds)
+    return units_per_step * steps * d.ws / slowest, slowest / steps * 1e3
+
+
 # ---- clocks ------------------------------------------------------------------------------
 
 class ClockSampler:
@@ -376,11 +384,9 @@ def run_samd(args, layers):
     wall = time.perf_counter() - t_wall
     clk = clocks.stop() if rank == 0 else None
     step_s = [a.elapsed_time(b) * 1e-3 for a, b in ev]
-    dev_time = d.max(sum(step_s))
+    value, ms_per_step = whole_job_rate(d, step_macs, args.steps, sum(step_s))
     if samd.samd_device_status() != 0:
         raise RuntimeError("a kernel recorded a timeout")
-    value = step_macs * args.steps * ws / dev_time
-    ms_per_step = dev_time / args.steps * 1e3
 
     # per-layer throughput (one graph per layer, replayed with events)
     by_layer = {}
