@@ -557,6 +557,11 @@ __device__ __forceinline__ void epilogue_row_spec(const ConvArgs &args, uint32_t
   uint32_t *row32 = reinterpret_cast<uint32_t *>(static_cast<uint8_t *>(args.packed_out) +
                                                  static_cast<size_t>(m) * args.out_wpr * (args.out_word64 ? 8 : 4)) +
                     ch0 / LH;
+  // 4-bit lanes: two 32-channel groups make one 32-byte store (a warp's
+  // 32-byte rows then cover whole 128-byte lines, in the L1 data path the
+  // MMAs' operand reads share)
+  const bool pair32 = NH == 4 && nvalid % 64 == 0 && (reinterpret_cast<uintptr_t>(row32) & 31) == 0;
+  uint32_t p0 = 0, p1 = 0, p2 = 0, p3 = 0;
   for (int col = 0; col < nvalid; col += 32) {
     uint32_t r[32];
     ptx::tmem_ld_32x32b_x32(taddr + col, r);
@@ -577,6 +582,16 @@ __device__ __forceinline__ void epilogue_row_spec(const ConvArgs &args, uint32_t
       }
       h[j] = OS ? w : w - bias_sum;
     }
+    if constexpr (NH == 4) {
+      if (pair32) {
+        if ((col & 32) == 0) {
+          p0 = h[0], p1 = h[1], p2 = h[2], p3 = h[3];
+        } else if (row_valid) {
+          ptx::st_global_v8(row32 + (col - 32) / LH, p0, p1, p2, p3, h[0], h[1], h[2], h[3]);
+        }
+        continue;
+      }
+    }
     if (!row_valid) continue;
     uint32_t *dst = row32 + col / LH;
     if (cnt < 32) {  // the last group of a channel count that is not a multiple of 32
@@ -587,6 +602,17 @@ __device__ __forceinline__ void epilogue_row_spec(const ConvArgs &args, uint32_t
           const int nl = cnt - c0 < LH ? cnt - c0 : LH;
           dst[j] = nl == LH ? h[j] : (h[j] & ((1u << (nl * OB)) - 1));
         }
+      }
+    } else if constexpr (NH == 8) {
+      if ((reinterpret_cast<uintptr_t>(dst) & 31) == 0) {
+        // one 32-byte store per row: with 32-byte rows a warp writes whole lines
+        ptx::st_global_v8(dst, h[0], h[1], h[2], h[3], h[4], h[5], h[6], h[7]);
+      } else if ((reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+        reinterpret_cast<uint4 *>(dst)[0] = make_uint4(h[0], h[1], h[2], h[3]);
+        reinterpret_cast<uint4 *>(dst)[1] = make_uint4(h[4], h[5], h[6], h[7]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < NH; ++j) dst[j] = h[j];
       }
     } else if constexpr (NH % 4 == 0) {
       if ((reinterpret_cast<uintptr_t>(dst) & 15) == 0) {

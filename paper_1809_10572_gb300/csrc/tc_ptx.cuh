@@ -105,6 +105,15 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+// 32-byte store (dst 32-byte aligned): a warp writing 32 consecutive 32-byte
+// rows covers eight whole 128-byte lines with one instruction.
+__device__ __forceinline__ void st_global_v8(void *dst, uint32_t v0, uint32_t v1, uint32_t v2, uint32_t v3,
+                                             uint32_t v4, uint32_t v5, uint32_t v6, uint32_t v7) {
+  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(dst), "r"(v0), "r"(v1), "r"(v2),
+               "r"(v3), "r"(v4), "r"(v5), "r"(v6), "r"(v7)
+               : "memory");
+}
+
 // ---- TMA -------------------------------------------------------------------
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void *tmap, int x, int y, uint32_t bar) {
