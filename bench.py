@@ -45,6 +45,9 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--layers", type=str, default="", help="comma-separated layer indices (profiling aid)")
+    ap.add_argument("--tiles-per-cta", type=int, default=0,
+                    help="samd_conv2d_set_min_tiles_per_cta for the step (0: 8 for the sweep's 32 concurrent "
+                         "small layers, else the library default)")
     ap.add_argument("--streams", type=int, default=8,
                     help="independent layers of a step run on this many streams (graph branches)")
     return ap.parse_args()
@@ -222,7 +225,8 @@ def workload_config(args, layers):
     return {"workload": desc, "layers": len(layers), "macs_per_step": workloads.total_macs(layers),
             "l2": "flushed before every step (512 MiB write, then 512 MiB read); inputs resident in HBM",
             "weights": "prepared once into the tensor-core operand layout (samd_conv2d_prepare), not in the step",
-            "launch": f"one CUDA graph per step; independent layers fanned out over {args.streams} streams",
+            "launch": f"one CUDA graph per step; independent layers fanned out over {args.streams} streams; "
+                      f"min 128-pixel tiles per CTA {args.tiles_per_cta or (8 if args.workload == 'sweep' else 4)}",
             "parallelism": f"replicas x{args.gpus}"}
 
 
@@ -323,6 +327,9 @@ def run_samd(args, layers):
     d = Dist("nccl")
     samd.load()
 
+    # the sweep's 32 small layers run concurrently: each keeps to a few SMs
+    tpc = args.tiles_per_cta or (8 if args.workload == "sweep" else 4)
+    samd.samd_conv2d_set_min_tiles_per_cta(tpc)
     built = build_layers(layers, dev)
     step_macs = workloads.total_macs(layers)
     flush_w = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)

@@ -162,9 +162,9 @@ typedef struct {
  * R*S*C * max|a| * max|w| reaches 2^24 and the weights have 5-8 bits, the
  * weights are split into two 4-bit digits (two exact accumulators per
  * output); if R*S*C * max|a| * 16 also reaches 2^24, SAMD_EUNSUP.
- * Scheduling: a layer of fewer than 4 x (SM count) 128-pixel tiles runs on
- * ceil(tiles / 4) SMs, so that independent layers issued on other streams
- * run beside it.
+ * Scheduling: a layer of fewer than T x (SM count) 128-pixel tiles runs on
+ * ceil(tiles / T) SMs (T = samd_conv2d_set_min_tiles_per_cta, default 4),
+ * so that independent layers issued on other streams run beside it.
  * Other limits (SAMD_EUNSUP): spacer 0 for fa and fw; R, S <= 16.
  * A kernel that gives up on a bounded wait leaves its outputs undefined and
  * records SAMD_ETIMEOUT for samd_device_status.
@@ -177,6 +177,14 @@ SAMD_API samd_status samd_conv2d(const samd_conv_desc *desc, samd_fmt fa, const 
  * output format (0 on error). The same size suffices for
  * samd_conv2d_prepare. */
 SAMD_API size_t samd_conv2d_workspace_size(const samd_conv_desc *desc, samd_fmt fa, samd_fmt fw);
+
+/* Minimum number of 128-pixel output tiles each SM works on in one
+ * convolution launch (process-wide, all devices, takes effect at the next
+ * launch). 1 spreads every layer over all SMs (lowest latency of a single
+ * layer); larger values leave SMs free for independent layers launched on
+ * other streams (higher throughput when several small layers run at once).
+ * Default 4. SAMD_EINVAL for values below 1 or above 1024. */
+SAMD_API samd_status samd_conv2d_set_min_tiles_per_cta(int tiles);
 
 /* Width in bits of the tensor-core operands samd_conv2d uses for this shape
  * and these formats: 8 (e4m3), 16 (fp16), or 0 if the convolution is

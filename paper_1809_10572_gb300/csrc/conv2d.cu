@@ -5,6 +5,7 @@
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
 
+#include <atomic>
 #include <cstring>
 #include <mutex>
 
@@ -168,7 +169,8 @@ long long max_abs(samd_fmt f) { return f.is_signed ? (1LL << (f.bits - 1)) : ((1
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 constexpr int kMaxHaloRows = 1024;
-constexpr int kMinTilesPerCta = 4;
+// minimum 128-pixel tiles per CTA of a launch (samd_conv2d_set_min_tiles_per_cta)
+std::atomic<int> g_min_tiles_per_cta{4};
 
 // Tiling, reduction order, operand type and exactness mode for one
 // convolution. fo.bits == 0 means no packed output. Returns SAMD_EUNSUP when
@@ -394,6 +396,8 @@ size_t conv2d_workspace_size(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw) 
   return best;
 }
 
+void conv2d_set_min_tiles_per_cta(int tiles) { conv::g_min_tiles_per_cta.store(tiles, std::memory_order_relaxed); }
+
 int conv2d_operand_bits(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw) {
   conv::Plan p;
   if (conv::make_plan(d, fa, fw, conv::none_fmt(), p) != SAMD_OK) return 0;
@@ -557,10 +561,11 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   a.g_stride = p.g_stride;
   a.off_e = p.off_e;
   a.off_bar = p.off_bar;
-  // a small layer keeps at least kMinTilesPerCta tiles per CTA, leaving SMs
-  // to independent layers issued on other streams
+  // a small layer keeps at least the set number of 128-pixel tiles per CTA,
+  // leaving SMs to independent layers issued on other streams
   const long long total_tiles = p.grid_m * p.nblocks;
-  const int min_tiles = kMinTilesPerCta / p.hv;  // at least 512 output positions per CTA
+  int min_tiles = g_min_tiles_per_cta.load(std::memory_order_relaxed) / p.hv;
+  if (min_tiles < 1) min_tiles = 1;
   long long ctas = (total_tiles + min_tiles - 1) / min_tiles;
   if (ctas > sm_count()) ctas = sm_count();
   dim3 grid(static_cast<unsigned>(ctas));

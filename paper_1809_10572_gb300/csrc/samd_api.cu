@@ -87,6 +87,12 @@ size_t samd_conv2d_workspace_size(const samd_conv_desc *d, samd_fmt fa, samd_fmt
   return conv2d_workspace_size(d, fa, fw);
 }
 
+samd_status samd_conv2d_set_min_tiles_per_cta(int tiles) {
+  if (tiles < 1 || tiles > 1024) return SAMD_EINVAL;
+  conv2d_set_min_tiles_per_cta(tiles);
+  return SAMD_OK;
+}
+
 int samd_conv2d_operand_bits(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw) {
   if (!d || !fmt_valid(fa) || !fmt_valid(fw) || fa.spacer != 0 || fw.spacer != 0) return 0;
   if (d->N < 0 || d->C < 1 || d->H < 1 || d->W < 1 || d->K < 1 || d->R < 1 || d->S < 1 || d->stride < 1 ||

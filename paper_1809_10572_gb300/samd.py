@@ -43,7 +43,7 @@ SAMD_NCHW, SAMD_NHWC = 0, 1
 OPS = {"add": SAMD_ADD, "sub": SAMD_SUB, "mul": SAMD_MUL, "relu": SAMD_RELU, "requant": SAMD_REQUANT}
 
 EXPORTED = ["samd_lanes_per_word", "samd_packed_words", "samd_pack", "samd_unpack", "samd_elementwise",
-            "samd_conv2d", "samd_conv2d_workspace_size", "samd_conv2d_operand_bits", "samd_conv2d_prepare", "samd_conv2d_prepared",
+            "samd_conv2d", "samd_conv2d_workspace_size", "samd_conv2d_operand_bits", "samd_conv2d_set_min_tiles_per_cta", "samd_conv2d_prepare", "samd_conv2d_prepared",
             "samd_conv2d_noalloc",
             "samd_maxpool2x2", "samd_device_status", "samd_status_str", "samd_version"]
 FMT_NONE = (0, 0, 0, 0)
@@ -95,6 +95,8 @@ def load(build_if_missing: bool = True):
     lib.samd_conv2d_workspace_size.restype = sz
     lib.samd_conv2d_operand_bits.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, samd_fmt]
     lib.samd_conv2d_operand_bits.restype = i32
+    lib.samd_conv2d_set_min_tiles_per_cta.argtypes = [i32]
+    lib.samd_conv2d_set_min_tiles_per_cta.restype = i32
     lib.samd_maxpool2x2.argtypes = [samd_fmt, vp, vp, i32, i32, i32, i32, i32, vp]
     lib.samd_maxpool2x2.restype = i32
     lib.samd_device_status.argtypes, lib.samd_device_status.restype = [c.POINTER(c.c_int), i32, vp], i32
@@ -168,6 +170,12 @@ def samd_elementwise(op, fa, a, b, fo, out, n, shift=0, saturate=0, stream=None)
 
 def samd_conv2d_workspace_size(desc: samd_conv_desc, fa: samd_fmt, fw: samd_fmt) -> int:
     return int(load().samd_conv2d_workspace_size(ctypes.byref(desc), fa, fw))
+
+
+def samd_conv2d_set_min_tiles_per_cta(tiles: int) -> None:
+    """Minimum 128-pixel tiles per SM of a convolution launch (1: spread each layer
+    over every SM; larger: leave SMs to layers running on other streams)."""
+    _check(load().samd_conv2d_set_min_tiles_per_cta(int(tiles)), "samd_conv2d_set_min_tiles_per_cta")
 
 
 def samd_conv2d_operand_bits(desc: samd_conv_desc, fa: samd_fmt, fw: samd_fmt) -> int:

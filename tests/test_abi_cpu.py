@@ -118,3 +118,10 @@ def test_conv_operand_type_query(lib):
     assert samd.samd_conv2d_operand_bits(d, samd.fmt(4, False, spacer=1), samd.fmt(4, True)) == 0
     assert samd.samd_conv2d_operand_bits(samd.ConvShape(1, 0, 8, 8, 16).desc(), samd.fmt(4, False),
                                          samd.fmt(4, True)) == 0
+
+
+def test_min_tiles_per_cta_setting(lib):
+    assert lib.samd_conv2d_set_min_tiles_per_cta(0) == samd.SAMD_EINVAL
+    assert lib.samd_conv2d_set_min_tiles_per_cta(1025) == samd.SAMD_EINVAL
+    assert lib.samd_conv2d_set_min_tiles_per_cta(8) == samd.SAMD_OK
+    assert lib.samd_conv2d_set_min_tiles_per_cta(4) == samd.SAMD_OK  # the default again
