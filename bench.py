@@ -395,7 +395,9 @@ def run_samd(args, layers):
     if samd.samd_device_status() != 0:
         raise RuntimeError("a kernel recorded a timeout")
 
-    # per-layer throughput (one graph per layer, replayed with events)
+    # per-layer throughput (one graph per layer, replayed with events; each
+    # layer alone, so with the library's default spread over the SMs)
+    samd.samd_conv2d_set_min_tiles_per_cta(4)
     by_layer = {}
     for b in built:
         g = torch.cuda.CUDAGraph()
@@ -513,14 +515,23 @@ def measure_e2e(built, step_macs, args, dev, ws, d):
     dev_in = [torch.empty_like(b["act"]) for b in built]
     h2d = sum(t.numel() * t.element_size() for t in host_in)
     d2h = sum(t.numel() * t.element_size() for t in host_out)
-    s = torch.cuda.current_stream()
+    # each layer's copy in, convolution and copy out run in order on one of
+    # the streams; the independent layers overlap across streams
+    streams = [torch.cuda.Stream(device=dev) for _ in range(max(1, args.streams))]
+    tpc = args.tiles_per_cta or (8 if args.workload == "sweep" else 4)
+
+    from paper_1809_10572_gb300 import samd
+    samd.samd_conv2d_set_min_tiles_per_cta(tpc)
 
     def step():
-        for b, hi, di, ho in zip(built, host_in, dev_in, host_out):
-            di.copy_(hi, non_blocking=True)
-            b["conv"](di, None, b["out"], b["shift"], stream=s)
-            ho.copy_(b["out"], non_blocking=True)
-        s.synchronize()
+        for i, (b, hi, di, ho) in enumerate(zip(built, host_in, dev_in, host_out)):
+            st = streams[i % len(streams)]
+            with torch.cuda.stream(st):
+                di.copy_(hi, non_blocking=True)
+                b["conv"](di, None, b["out"], b["shift"], stream=st)
+                ho.copy_(b["out"], non_blocking=True)
+        for st in streams:
+            st.synchronize()
 
     for _ in range(max(1, args.warmup)):
         step()
@@ -530,8 +541,9 @@ def measure_e2e(built, step_macs, args, dev, ws, d):
         step()
     el = d.max(time.perf_counter() - t0)
     return {"value": step_macs * args.steps * ws / el, "unit": "MAC/s", "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "how": "per layer: pinned H2D of packed act, samd_conv2d_prepared, "
-                                               "pinned D2H of packed output; sync per step"}
+            "d2h_bytes_per_step": d2h, "how": "per layer on one of the step's streams: pinned H2D of its packed "
+                                               "input, samd_conv2d_prepared, pinned D2H of its packed output; "
+                                               "host waits for every stream each step"}
 
 
 def main():
