@@ -248,6 +248,16 @@ SAMD_API samd_status samd_maxpool2x2(samd_fmt f, const void *in, void *out, int 
  */
 SAMD_API samd_status samd_device_status(int *status, int reset, samd_stream_t stream);
 
+/*
+ * samd_selftest_wait_timeout: exercises the failure path of the bounded waits
+ * without faulting the GPU. Launches one block on `stream` whose thread waits
+ * on an mbarrier phase that nothing completes; after limit_ns nanoseconds
+ * (1000 .. 2e9, else SAMD_EINVAL) the wait gives up and records
+ * SAMD_ETIMEOUT in the sticky status read by samd_device_status, as a
+ * convolution role that gives up does. The context stays usable. Asynchronous.
+ */
+SAMD_API samd_status samd_selftest_wait_timeout(uint64_t limit_ns, samd_stream_t stream);
+
 /* A static string naming the status. */
 SAMD_API const char *samd_status_str(samd_status s);
 

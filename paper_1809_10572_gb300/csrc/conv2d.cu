@@ -609,6 +609,25 @@ samd_status conv2d_nhwc_noalloc(const samd_conv_desc *d, samd_fmt fa, const void
   return conv2d_nhwc(d, fa, act, fw, wt, acc_out, fo, packed_out, shift, scratch, kNoallocScratchBytes, s);
 }
 
+// One thread waits, bounded by limit_ns, on an mbarrier phase that nothing
+// completes; the wait runs out and the thread records SAMD_ETIMEOUT exactly as
+// a convolution role that gives up does. Nothing is in flight when it returns.
+__global__ void wait_timeout_kernel(uint64_t limit_ns) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(ptx::smem_addr(&bar), 1);
+    ptx::fence_barrier_init();
+    int quiet = 0;
+    if (!ptx::mbar_wait_bounded(ptx::smem_addr(&bar), 0, &quiet, limit_ns))
+      atomicOr(&g_conv_status, static_cast<int>(SAMD_ETIMEOUT));
+  }
+}
+
+cudaError_t selftest_wait_timeout(uint64_t limit_ns, cudaStream_t s) {
+  wait_timeout_kernel<<<1, 32, 0, s>>>(limit_ns);
+  return cudaGetLastError();
+}
+
 cudaError_t read_device_status(int *status, int reset, cudaStream_t s) {
   int v = 0;
   cudaError_t e = cudaMemcpyFromSymbolAsync(&v, g_conv_status, sizeof(int), 0, cudaMemcpyDeviceToHost, s);

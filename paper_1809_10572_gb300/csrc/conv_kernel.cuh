@@ -778,7 +778,7 @@ __device__ __forceinline__ void epilogue_row(const ConvArgs &args, uint32_t tadd
   }
 }
 
-// Issues `ksteps` (1..4) MMAs of one operand row as straight-line code.
+// One MMA.
 template <bool FP8>
 __device__ __forceinline__ void mma_op(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
   if constexpr (FP8)
@@ -796,6 +796,7 @@ __device__ __forceinline__ void mma_kstep(uint32_t d, uint32_t dn, uint64_t a, u
   if constexpr (HV == 2) mma_op<FP8>(d + dn, a + ah, b, idesc, acc);
 }
 
+// Issues `ksteps` (1..4) k-steps of one operand row as straight-line code.
 template <bool FP8, int HV>
 __device__ __forceinline__ void mma_ksteps(int ksteps, uint32_t d, uint32_t dn, uint64_t a, uint64_t ah, uint64_t b,
                                            uint32_t idesc, uint32_t acc) {
@@ -879,7 +880,6 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
   constexpr int WC = U::WC;
   using St = Staging<W, WC>;
   extern __shared__ uint8_t smem_raw[];
-  __shared__ int s_skip;
   uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
 
   const int STB = args.stages;  // weight tiles in flight (or resident)
@@ -902,9 +902,8 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
 
   volatile int *status = args.status;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (threadIdx.x == 0) s_skip = *status;
-  __syncthreads();
-  if (s_skip) return;
+  // No global read precedes the setup barrier: a failure recorded by an
+  // earlier launch is seen by the first wait that has to wait.
   if (warp == 0) {
     ptx::tmem_alloc(ptx::smem_addr(tmem_holder), args.tmem_cols);
     ptx::tmem_relinquish();
@@ -925,6 +924,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     ptx::mbar_init(drain_bar, 1);
     ptx::fence_barrier_init();
   }
+  __syncwarp();  // every warp reaches the barrier converged (bar.sync counts whole warps)
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
@@ -939,11 +939,14 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     if (lane == 0) {
       // ---- weight tiles ----
       ptx::prefetch_tmap(&tmap_b);
+      int quiet = 0;  // the waits below end only when the copies land (or time out)
       if (resident) {
         for (int c = 0; c < nchunks; ++c) {
           ptx::mbar_arrive_expect_tx(full_b(c), b_bytes);
           ptx::tma_load_2d(ptx::smem_addr(sB + c * b_bytes), &tmap_b, c * BK, 0, full_b(c));
         }
+        // the CTA does not exit with a copy in flight, whatever the other roles do
+        for (int c = 0; c < nchunks; ++c) ptx::mbar_wait_bounded(full_b(c), 0, &quiet, kWaitLimitNs);
       } else {
         long long cb = 0, issued_from = 0;
         for (long long tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
@@ -962,7 +965,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         }
         if (!ok) {  // leave no copy in flight: wait (bounded) for the last ring's worth
           for (long long k = (cb - STB > issued_from ? cb - STB : issued_from); k < cb; ++k)
-            ptx::mbar_wait_bounded(full_b(static_cast<int>(k % STB)), static_cast<uint32_t>((k / STB) & 1), status,
+            ptx::mbar_wait_bounded(full_b(static_cast<int>(k % STB)), static_cast<uint32_t>((k / STB) & 1), &quiet,
                                    kWaitLimitNs / 10);
         }
       }
@@ -1240,16 +1243,24 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     const int row = quad * 32 + lane;
     constexpr int kTileStep = HV == 2 ? 1 : 2;
     long long i = HV == 2 ? 0 : set;
-    for (long long tile = first_tile + (HV == 2 ? 0 : set) * tile_step; tile < total_tiles;
-         tile += kTileStep * tile_step, i += kTileStep) {
+    // The first pass over the first tile runs with its stores off and without
+    // waiting for the accumulator (whatever it reads is discarded): the row
+    // epilogue is the largest code of the kernel, and this way its
+    // instructions are fetched while the first tile is being computed rather
+    // than after it.
+    bool warm = true;
+    for (long long tile = first_tile + (HV == 2 ? 0 : set) * tile_step; tile < total_tiles;) {
       const int acc_i = HV == 2 ? static_cast<int>(i & 1) : set;  // accumulator of this tile
-      bool w_ok = true;
-      if (lane == 0) w_ok = ptx::mbar_wait_bounded(accfull(acc_i), static_cast<uint32_t>((i >> 1) & 1), status, kWaitLimitNs);
-      if (!__shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0)) {
-        ok = false;
-        break;
+      if (!warm) {
+        bool w_ok = true;
+        if (lane == 0)
+          w_ok = ptx::mbar_wait_bounded(accfull(acc_i), static_cast<uint32_t>((i >> 1) & 1), status, kWaitLimitNs);
+        if (!__shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0)) {
+          ok = false;
+          break;
+        }
+        ptx::tc_fence_after();
       }
-      ptx::tc_fence_after();
       const uint32_t tl = static_cast<uint32_t>(tile);
       const uint32_t nbu = fdiv(tl, args.fd_gm);
       const int nb = static_cast<int>(nbu);
@@ -1271,13 +1282,20 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       }
       const uint32_t taddr = tmem_base + static_cast<uint32_t>((acc_i * HV + (HV == 2 ? set : 0)) * args.mma_n) +
                              (static_cast<uint32_t>(quad * 32) << 16);
-      epilogue_row(args, taddr, valid, m, nb);
+      epilogue_row(args, taddr, valid && !warm, m, nb);
+      if (warm) {
+        warm = false;
+        continue;
+      }
       ptx::tc_fence_before();
       __syncwarp();
       if (lane == 0) ptx::mbar_arrive(accempty(acc_i));
+      tile += kTileStep * tile_step;
+      i += kTileStep;
     }
   }
 
+  __syncwarp();
   ptx::tc_fence_before();
   __syncthreads();
   if (warp == 0) {

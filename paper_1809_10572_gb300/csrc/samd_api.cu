@@ -194,6 +194,11 @@ samd_status samd_device_status(int *status, int reset, samd_stream_t stream) {
   return from_cuda(read_device_status(status, reset, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+samd_status samd_selftest_wait_timeout(uint64_t limit_ns, samd_stream_t stream) {
+  if (limit_ns < 1000ull || limit_ns > 2000000000ull) return SAMD_EINVAL;
+  return from_cuda(selftest_wait_timeout(limit_ns, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 const char *samd_status_str(samd_status s) {
   switch (s) {
     case SAMD_OK: return "SAMD_OK";

@@ -96,4 +96,5 @@ constexpr size_t kNoallocScratchBytes = size_t(8) << 20;  // static scratch of s
 samd_status conv2d_nhwc_noalloc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
                                 int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, cudaStream_t s);
 cudaError_t read_device_status(int *status, int reset, cudaStream_t s);
+cudaError_t selftest_wait_timeout(uint64_t limit_ns, cudaStream_t s);
 }  // namespace samd

@@ -45,7 +45,7 @@ OPS = {"add": SAMD_ADD, "sub": SAMD_SUB, "mul": SAMD_MUL, "relu": SAMD_RELU, "re
 EXPORTED = ["samd_lanes_per_word", "samd_packed_words", "samd_pack", "samd_unpack", "samd_elementwise",
             "samd_conv2d", "samd_conv2d_workspace_size", "samd_conv2d_operand_bits", "samd_conv2d_set_min_tiles_per_cta", "samd_conv2d_prepare", "samd_conv2d_prepared",
             "samd_conv2d_noalloc",
-            "samd_maxpool2x2", "samd_device_status", "samd_status_str", "samd_version"]
+            "samd_maxpool2x2", "samd_device_status", "samd_selftest_wait_timeout", "samd_status_str", "samd_version"]
 FMT_NONE = (0, 0, 0, 0)
 
 
@@ -100,6 +100,7 @@ def load(build_if_missing: bool = True):
     lib.samd_maxpool2x2.argtypes = [samd_fmt, vp, vp, i32, i32, i32, i32, i32, vp]
     lib.samd_maxpool2x2.restype = i32
     lib.samd_device_status.argtypes, lib.samd_device_status.restype = [c.POINTER(c.c_int), i32, vp], i32
+    lib.samd_selftest_wait_timeout.argtypes, lib.samd_selftest_wait_timeout.restype = [c.c_uint64, vp], i32
     lib.samd_status_str.argtypes, lib.samd_status_str.restype = [i32], c.c_char_p
     lib.samd_version.argtypes, lib.samd_version.restype = [], c.c_char_p
     _lib = lib
@@ -227,6 +228,10 @@ def samd_device_status(reset: bool = False, stream=None) -> int:
     v = ctypes.c_int(0)
     _check(load().samd_device_status(ctypes.byref(v), int(reset), _stream(stream)), "samd_device_status")
     return v.value
+
+
+def samd_selftest_wait_timeout(limit_ns: int, stream=None) -> None:
+    _check(load().samd_selftest_wait_timeout(limit_ns, _stream(stream)), "samd_selftest_wait_timeout")
 
 
 def samd_version() -> str:

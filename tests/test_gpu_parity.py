@@ -240,3 +240,20 @@ def test_conv_misaligned_pointer_rejected(samd_lib):
     with pytest.raises(samd.SamdError) as e:
         samd.samd_conv2d(shape.desc(), fa, a_w, fw, w_w, acc[1:], None, None, 0, ws)
     assert e.value.status == samd.SAMD_EALIGN
+
+
+def test_bounded_wait_timeout_is_recorded_and_the_context_survives(samd_lib):
+    # a wait on an mbarrier phase that nothing completes runs out after 2 ms
+    # and records SAMD_ETIMEOUT; no trap, the context stays usable
+    assert samd.samd_device_status(reset=True) in (samd.SAMD_OK, samd.SAMD_ETIMEOUT)
+    assert samd.samd_device_status() == samd.SAMD_OK
+    samd.samd_selftest_wait_timeout(2_000_000)
+    torch.cuda.synchronize()
+    assert samd.samd_device_status(reset=True) == samd.SAMD_ETIMEOUT
+    assert samd.samd_device_status() == samd.SAMD_OK
+    # a convolution after the reset is bit-exact and leaves the status clean
+    shape = samd.ConvShape(2, 24, 10, 9, 32)
+    run_conv_check(shape, 4, False, 4, True, fo_t=(4, False, 0, 32), seed=11)
+    with pytest.raises(samd.SamdError) as e:
+        samd.samd_selftest_wait_timeout(10)
+    assert e.value.status == samd.SAMD_EINVAL
