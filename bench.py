@@ -30,6 +30,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 L2_FLUSH_BYTES = 512 << 20  # > 129 MB L2
+L2_BYTES = 129 * 10**6
 METRIC = "effective int MAC/s for b-bit conv2d vs bit width (fraction of int8 TC peak); packed-op GB/s"
 
 
@@ -48,6 +49,9 @@ def parse_args():
     ap.add_argument("--tiles-per-cta", type=int, default=0,
                     help="samd_conv2d_set_min_tiles_per_cta for the step (0: 8 for the sweep's 32 concurrent "
                          "small layers, else the library default)")
+    ap.add_argument("--l2", default="rotate", choices=["rotate", "flush"],
+                    help="keep a step's data out of L2 by cycling through sets of inputs larger than L2 in "
+                         "total (rotate), or by flushing L2 before every step (flush)")
     ap.add_argument("--streams", type=int, default=8,
                     help="independent layers of a step run on this many streams (graph branches)")
     return ap.parse_args()
@@ -223,10 +227,15 @@ def workload_config(args, layers):
         "conv1x": "3x3 conv N1 C16->16 32x32, u4 x s4, 64-bit words",
     }[args.workload]
     return {"workload": desc, "layers": len(layers), "macs_per_step": workloads.total_macs(layers),
-            "l2": "flushed before every step (512 MiB write, then 512 MiB read); inputs resident in HBM",
+            "l2": ("inputs larger than L2: independent sets of packed inputs, prepared weights and outputs, "
+                   "together at least twice the L2, used in turn (one set per step), no flush; "
+                   "value_l2_flushed: one set with L2 flushed (512 MiB write + 512 MiB read) before every step"
+                   if args.l2 == "rotate" else
+                   "flushed before every step (512 MiB write, then 512 MiB read); inputs resident in HBM"),
             "weights": "prepared once into the tensor-core operand layout (samd_conv2d_prepare), not in the step",
             "launch": f"one CUDA graph per step; independent layers fanned out over {args.streams} streams; "
-                      f"min 128-pixel tiles per CTA {args.tiles_per_cta or (8 if args.workload == 'sweep' else 4)}",
+                      f"each CTA at least {args.tiles_per_cta or (8 if args.workload == 'sweep' else 4)} reference tiles "
+                      f"of work (samd_conv2d_set_min_tiles_per_cta)",
             "parallelism": f"replicas x{args.gpus}"}
 
 
@@ -332,6 +341,16 @@ def run_samd(args, layers):
     samd.samd_conv2d_set_min_tiles_per_cta(tpc)
     built = build_layers(layers, dev)
     step_macs = workloads.total_macs(layers)
+    # Between timed steps no step may find its data in L2. The step works on
+    # one of R independent sets of inputs, prepared weights and outputs, the
+    # next set each step, with R x (bytes of a set) at least twice the L2:
+    # when a set comes round again, more than an L2's worth of other data has
+    # passed through since. (--l2 flush keeps one set and flushes L2 instead;
+    # the line reports that number too.)
+    set_bytes = sum(t.numel() * t.element_size() for b in built
+                    for t in (b["act"], b["out"], b["conv"].prepared))
+    n_sets = max(1, -(-2 * L2_BYTES // set_bytes)) if args.l2 == "rotate" else 1
+    sets = [built] + [build_layers(layers, dev) for _ in range(n_sets - 1)]
     flush_w = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     flush_r = torch.ones(L2_FLUSH_BYTES // 8, dtype=torch.int64, device=dev)
 
@@ -345,56 +364,75 @@ def run_samd(args, layers):
     stream = torch.cuda.Stream(device=dev)
     side = [torch.cuda.Stream(device=dev) for _ in range(max(1, args.streams))]
 
-    def step_calls(main):
+    def step_calls(main, bs):
         # the layers of the workload are independent: fan them out over the
         # side streams and join them back into `main`
         for sd in side:
             sd.wait_stream(main)
-        for i, b in enumerate(built):
+        for i, b in enumerate(bs):
             b["conv"](b["act"], None, b["out"], b["shift"], stream=side[i % len(side)])
         for sd in side:
             main.wait_stream(sd)
 
     # first calls outside any capture (kernel attributes, tensor-map entry point)
     with torch.cuda.stream(stream):
-        step_calls(stream)
+        step_calls(stream, built)
     torch.cuda.synchronize()
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph, stream=stream):
-        step_calls(torch.cuda.current_stream())
+    graphs = []
+    for bs in sets:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            step_calls(torch.cuda.current_stream(), bs)
+        graphs.append(g)
     torch.cuda.synchronize()
     if samd.samd_device_status() != 0:
         raise RuntimeError("a kernel recorded a timeout")
 
-    # warm-up
-    for _ in range(args.warmup):
-        flush()
-        graph.replay()
-    torch.cuda.synchronize()
+    def timed_steps(use_flush, sample_clocks):
+        """K steps after W warm-up steps; with use_flush one set and an L2
+        flush before every step (outside the events), else the sets in turn."""
+        gs = graphs[:1] if use_flush else graphs
+        for w in range(args.warmup):
+            if use_flush:
+                flush()
+            gs[w % len(gs)].replay()
+        torch.cuda.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        clocks = ClockSampler(local)
+        if sample_clocks and rank == 0:
+            clocks.start()
+        d.barrier()
+        torch.cuda.synchronize()
+        t_wall = time.perf_counter()
+        cur = torch.cuda.current_stream()
+        for i in range(args.steps):
+            if use_flush:
+                flush()
+            ev[i][0].record(cur)
+            gs[(args.warmup + i) % len(gs)].replay()
+            ev[i][1].record(cur)
+        torch.cuda.synchronize()
+        d.barrier()
+        wall_s = time.perf_counter() - t_wall
+        clk_s = clocks.stop() if sample_clocks and rank == 0 else None
+        if samd.samd_device_status() != 0:
+            raise RuntimeError("a kernel recorded a timeout")
+        return [a.elapsed_time(b) * 1e-3 for a, b in ev], wall_s, clk_s
 
-    # timed region: K steps, L2 flushed between steps (outside the events)
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-    clocks = ClockSampler(local)
-    if rank == 0:
-        clocks.start()
-    d.barrier()
-    torch.cuda.synchronize()
-    t_wall = time.perf_counter()
-    cur = torch.cuda.current_stream()
-    for i in range(args.steps):
-        flush()
-        ev[i][0].record(cur)
-        graph.replay()
-        ev[i][1].record(cur)
-    torch.cuda.synchronize()
-    d.barrier()
-    wall = time.perf_counter() - t_wall
-    clk = clocks.stop() if rank == 0 else None
-    step_s = [a.elapsed_time(b) * 1e-3 for a, b in ev]
+    # timed region
+    step_s, wall, clk = timed_steps(args.l2 == "flush", True)
     value, ms_per_step = whole_job_rate(d, step_macs, args.steps, sum(step_s))
-    if samd.samd_device_status() != 0:
-        raise RuntimeError("a kernel recorded a timeout")
+    if args.l2 == "rotate":  # the same step with one set and an L2 flush before every step
+        flushed_s, _, _ = timed_steps(True, False)
+        value_flushed, _ = whole_job_rate(d, step_macs, args.steps, sum(flushed_s))
+    else:
+        value_flushed = value
+    l2_note = (f"inputs larger than L2: {n_sets} sets of packed inputs, prepared weights and outputs "
+               f"({n_sets} x {set_bytes / 1e6:.1f} MB) used in turn, one set per step, no flush"
+               if args.l2 == "rotate" else
+               "flushed before every step (512 MiB write, then 512 MiB read); inputs resident in HBM")
 
+    cur = torch.cuda.current_stream()
     # per-layer throughput (one graph per layer, replayed with events; each
     # layer alone, so with the library's default spread over the SMs)
     samd.samd_conv2d_set_min_tiles_per_cta(4)
@@ -441,7 +479,8 @@ def run_samd(args, layers):
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "e4m3 or f16 operands -> f32 tensor-core accumulation of exact integers (b-bit packed lanes)",
         "data": "synthetic",
-        "config": workload_config(args, layers), "wall_s_timed_region": wall,
+        "config": workload_config(args, layers), "l2_sets": l2_note, "value_l2_flushed": value_flushed,
+        "wall_s_timed_region": wall,
         "gpu_launches": args.steps * len(built),
         "roofline": roofline,
     }

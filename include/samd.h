@@ -162,9 +162,10 @@ typedef struct {
  * R*S*C * max|a| * max|w| reaches 2^24 and the weights have 5-8 bits, the
  * weights are split into two 4-bit digits (two exact accumulators per
  * output); if R*S*C * max|a| * 16 also reaches 2^24, SAMD_EUNSUP.
- * Scheduling: a layer of fewer than T x (SM count) 128-pixel tiles runs on
- * ceil(tiles / T) SMs (T = samd_conv2d_set_min_tiles_per_cta, default 4),
- * so that independent layers issued on other streams run beside it.
+ * Scheduling: a layer with less than T x (SM count) reference tiles of work
+ * (T = samd_conv2d_set_min_tiles_per_cta, default 4) runs on fewer SMs, each
+ * doing at least T reference tiles, so that independent layers issued on
+ * other streams run beside it.
  * Other limits (SAMD_EUNSUP): spacer 0 for fa and fw; R, S <= 16.
  * A kernel that gives up on a bounded wait leaves its outputs undefined and
  * records SAMD_ETIMEOUT for samd_device_status.
@@ -178,12 +179,15 @@ SAMD_API samd_status samd_conv2d(const samd_conv_desc *desc, samd_fmt fa, const 
  * samd_conv2d_prepare. */
 SAMD_API size_t samd_conv2d_workspace_size(const samd_conv_desc *desc, samd_fmt fa, samd_fmt fw);
 
-/* Minimum number of 128-pixel output tiles each SM works on in one
- * convolution launch (process-wide, all devices, takes effect at the next
- * launch). 1 spreads every layer over all SMs (lowest latency of a single
- * layer); larger values leave SMs free for independent layers launched on
- * other streams (higher throughput when several small layers run at once).
- * Default 4. SAMD_EINVAL for values below 1 or above 1024. */
+/* Minimum work each SM does in one convolution launch, T, in reference
+ * tiles: 128 output positions of a 3x3 convolution over 64 input and 64
+ * output channels (4.7 M multiply-adds). A layer whose 128-position tiles
+ * carry w times that work gets floor(T / w) tiles per SM, at least one
+ * (process-wide, all devices, takes effect at the next launch). 1 spreads
+ * every layer over all SMs (lowest latency of a single layer); larger values
+ * leave SMs free for independent layers launched on other streams (higher
+ * throughput when several small layers run at once). Default 4.
+ * SAMD_EINVAL for values below 1 or above 1024. */
 SAMD_API samd_status samd_conv2d_set_min_tiles_per_cta(int tiles);
 
 /* Width in bits of the tensor-core operands samd_conv2d uses for this shape

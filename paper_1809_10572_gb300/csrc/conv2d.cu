@@ -561,10 +561,17 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   a.g_stride = p.g_stride;
   a.off_e = p.off_e;
   a.off_bar = p.off_bar;
-  // a small layer keeps at least the set number of 128-pixel tiles per CTA,
-  // leaving SMs to independent layers issued on other streams
+  // A small layer gives each CTA at least T reference tiles of work (T from
+  // samd_conv2d_set_min_tiles_per_cta; a reference tile is 128 positions of
+  // a 3x3 convolution over 64 input and 64 output channels: 9 operand rows of
+  // 64 positions, 64 MMA columns), leaving SMs to independent layers issued
+  // on other streams. A tile of this layer weighs hv * nchunks * mma_n of
+  // those 9 * 64, so layers with long reductions or many output channels
+  // spread over more SMs.
   const long long total_tiles = p.grid_m * p.nblocks;
-  int min_tiles = g_min_tiles_per_cta.load(std::memory_order_relaxed) / p.hv;
+  const long long ref_work = static_cast<long long>(g_min_tiles_per_cta.load(std::memory_order_relaxed)) * 9 * 64;
+  const long long tile_work = static_cast<long long>(p.hv) * p.nchunks * p.mma_n;
+  long long min_tiles = ref_work / tile_work;
   if (min_tiles < 1) min_tiles = 1;
   long long ctas = (total_tiles + min_tiles - 1) / min_tiles;
   if (ctas > sm_count()) ctas = sm_count();
