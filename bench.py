@@ -19,6 +19,8 @@ C ABI from pinned host buffers; the CPU oracle timed on the host cores.
 from __future__ import annotations
 
 import argparse
+import glob
+import hashlib
 import json
 import os
 import statistics
@@ -324,6 +326,33 @@ def time_packed_ops(dev, flush):
     return res
 
 
+def csrc_digest():
+    """sha256 over the kernel sources (file names and contents)."""
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_1809_10572_gb300", "csrc")
+    for f in sorted(glob.glob(os.path.join(csrc, "*.cu")) + glob.glob(os.path.join(csrc, "*.cuh"))):
+        h.update(os.path.basename(f).encode())
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def measured_traffic(args):
+    """DRAM bytes per conv launch of the sweep step from the committed ncu
+    summary, if the kernel sources are still the ones it measured."""
+    if args.workload != "sweep" or args.layers:
+        return None, "measured for the full sweep step only"
+    try:
+        with open(os.path.join(ROOT, "profiles", "conv_kernel_sweep_traffic.json")) as fh:
+            rec = json.load(fh)
+    except (OSError, ValueError):
+        return None, "no ncu traffic summary"
+    if rec.get("csrc_sha256") != csrc_digest():
+        return None, "kernel sources changed since the ncu traffic capture"
+    return rec["dram_bytes_per_launch"], ("ncu dram__bytes_read.sum + dram__bytes_write.sum, mean over the step's "
+                                          f"{rec['launches']} launches (profiles/conv_kernel_sweep_traffic.md)")
+
+
 def run_samd(args, layers):
     import torch
 
@@ -468,8 +497,10 @@ def run_samd(args, layers):
     step_peak = 2.0 * step_macs / ideal_s / 1e12
     n_e4m3 = sum(1 for b in built if b["operand_bits"] == 8)
     achieved_tflops = 2.0 * step_macs / (ms_per_step * 1e-3) / 1e12
+    traffic, traffic_note = measured_traffic(args)
     roofline = {"kernel": "conv_kernel", "bound": "tensor", "achieved": achieved_tflops, "peak": step_peak,
-                "unit": "TFLOP/s", "frac": achieved_tflops / step_peak, "traffic": None,
+                "unit": "TFLOP/s", "frac": achieved_tflops / step_peak, "traffic": traffic,
+                "traffic_note": traffic_note,
                 "peak_source": f"{peak_src} bf16 burst {bf16_peak:.1f} TFLOP/s for fp16 layers, x2 for e4m3 layers "
                                f"({n_e4m3} of {len(built)} layers), MAC-weighted",
                 "note": "achieved = 2 x direct-conv MACs of the step / step time (all launches are the conv kernel)"}
