@@ -152,6 +152,8 @@ struct Plan {
   int hv;         // tile of hv halves of 128 output positions
   int row_bytes;  // operand row: 64 (e4m3) or 128 (fp16) bytes
   int wpr, words_total, La, WC, nchunks, Kpad, NBc, n_mma, mma_n, split, nblocks, stages, Ho, Wo, gather_vec;
+  int gather_win;  // 1x1 gather through 16-byte windows (AGather::issue_win)
+  int g_row;       // gather staging row pitch in bytes
   int halo, Hv, Wp, nck, taps;
   int nseg, seg_rows, seg_used, row_step;  // halo geometry (see ConvArgs)
   long long grid_m;                        // 128-position tiles along the output
@@ -219,6 +221,15 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
   const int srow = (chunk_bytes + 15) / 16 * 16;  // Staging::kRowBytes
   const int vec = chunk_bytes % 16 == 0 ? 16 : (chunk_bytes % 8 == 0 ? 8 : wb);
   p.gather_vec = (p.wpr % p.WC == 0) && ((static_cast<long long>(p.wpr) * wb) % vec == 0) ? 1 : 0;
+  // A 1x1 layer whose chunks are not whole aligned vectors copies each
+  // chunk through the 16-byte-aligned window around it: one more 16-byte
+  // piece than the chunk, and an odd number of pieces per staging row, so
+  // that a quarter-warp's 16-byte accesses to eight rows hit distinct banks.
+  p.gather_win = (!p.gather_vec && d->R == 1 && d->S == 1) ? 1 : 0;
+  int win_pieces = srow / 16 + 1;
+  if (win_pieces % 2 == 0) ++win_pieces;
+  const int grow = p.gather_win ? win_pieces * 16 : srow;
+  p.g_row = grow;
   p.b_bytes = static_cast<uint32_t>(p.mma_n) * p.row_bytes;  // a multiple of 1024
   const size_t bst = p.b_bytes;
   const size_t e_bytes = 0;  // the epilogue packs in registers
@@ -299,7 +310,7 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
       return true;
     }
     const size_t tile_bytes = static_cast<size_t>(bmt) * p.row_bytes;
-    const size_t group_slots = static_cast<size_t>(kGatherDepth) * BM * srow;  // one producer group's ring
+    const size_t group_slots = static_cast<size_t>(kGatherDepth) * BM * grow;  // one producer group's ring
     for (int sta = 4; sta >= 2; --sta) {
       const size_t fixed = sta * tile_bytes + 2 * group_slots + e_bytes + 1024;
       if (fixed + 2 * bst + bar_bytes(2, sta) > kBudget) continue;
@@ -516,6 +527,9 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   a.grid_m = p.grid_m;
   a.nblocks = p.nblocks;
   a.gather_vec = p.gather_vec;
+  a.gather_win = p.gather_win;
+  a.g_row = p.g_row;
+  a.act_bytes = static_cast<long long>(d->N) * d->H * d->W * p.wpr * (fa.word_bits / 8);
   a.tmem_cols = p.tmem_cols;
   a.out_bits = packed_out ? fo.bits : 8;
   a.out_signed = packed_out ? fo.is_signed : 1;

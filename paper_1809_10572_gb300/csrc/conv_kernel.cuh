@@ -154,6 +154,9 @@ struct ConvArgs {
   long long grid_m; // 128-position tiles along the output
   int nblocks;      // channel blocks
   int gather_vec;   // AGather::vec
+  int gather_win;   // AGather::issue_win (1x1 layers whose chunks are not aligned vectors)
+  int g_row;        // GATHER staging row pitch in bytes
+  long long act_bytes;  // bytes of the activation tensor (the windows stop at its end)
   uint32_t tmem_cols;
   int out_bits, out_signed, out_lane_w, out_L, out_word64, out_wpr;
   int out_fast;     // output lanes per word when they divide 32 (whole words per 32 channels), else 0
@@ -371,6 +374,42 @@ __device__ __forceinline__ void load_staged(const uint8_t *src, W (&cur)[WC]) {
   }
 }
 
+// 16-byte pieces that cover one chunk from the 16-byte boundary at or below
+// its first byte (the chunk then starts o bytes into the staged row, o < 16).
+template <typename W, int WC>
+constexpr int kWinPieces = (WC * static_cast<int>(sizeof(W)) + 15) / 16 + 1;
+
+// Reads a chunk staged through its 16-byte window (AGather::issue_win): the
+// chunk starts o4 32-bit units into the row; words from nw on are zero.
+template <typename W, int WC>
+__device__ __forceinline__ void load_window(const uint8_t *row, int o4, int nw, W (&cur)[WC]) {
+  constexpr int kU = WC * static_cast<int>(sizeof(W)) / 4;  // 32-bit units of a chunk
+  constexpr int kV = (kU + 3 + 3) / 4;                       // 16-byte reads covering kU + 3 units
+  static_assert(kV <= kWinPieces<W, WC>, "the window holds every unit read");
+  uint32_t u[4 * kV];
+#pragma unroll
+  for (int v = 0; v < kV; ++v) {
+    const uint4 q = *reinterpret_cast<const uint4 *>(row + 16 * v);
+    u[4 * v] = q.x, u[4 * v + 1] = q.y, u[4 * v + 2] = q.z, u[4 * v + 3] = q.w;
+  }
+  // shift down by o4 units: by one unit, then by two
+  uint32_t s1[kU + 2];
+#pragma unroll
+  for (int i = 0; i < kU + 2; ++i) s1[i] = (o4 & 1) ? u[i + 1] : u[i];
+  const int nu = nw * static_cast<int>(sizeof(W)) / 4;
+#pragma unroll
+  for (int i = 0; i < kU; ++i) {
+    uint32_t x = (o4 & 2) ? s1[i + 2] : s1[i];
+    if (i >= nu) x = 0u;
+    if constexpr (sizeof(W) == 4)
+      cur[i] = x;
+    else if (i & 1)
+      cur[i / 2] |= static_cast<W>(x) << 32;
+    else
+      cur[i / 2] = x;
+  }
+}
+
 // Gathers the packed words of one pixel's chunk into shared memory with
 // cp.async: word kw of the reduction is word (kw mod wpr) of the input pixel
 // at tap kw / wpr; taps outside the image and words past the end are
@@ -413,6 +452,30 @@ struct AGather {
         px = pixel(tap, valid);
       }
     }
+  }
+
+  // 1x1 layers (one tap): the chunk's bytes are copied as the 16-byte pieces
+  // of the aligned window around them, so that every copy is 16 bytes wide
+  // whatever the pixel's alignment. Pieces past the chunk are zero-filled;
+  // a piece that reaches past the end of the activation tensor (act_end)
+  // copies only the bytes before it. Returns the chunk's offset into the
+  // staged row in 32-bit units (load_window). act is 16-byte aligned.
+  __device__ __forceinline__ int issue_win(int chunk, uint32_t dst, uintptr_t act_end) const {
+    const int kw0 = chunk * WC;
+    const int nw = words_total - kw0 < WC ? words_total - kw0 : WC;
+    bool valid;
+    const W *px = pixel(0, valid);
+    const uintptr_t a = valid ? reinterpret_cast<uintptr_t>(px + kw0) : reinterpret_cast<uintptr_t>(act);
+    const uintptr_t a0 = a & ~static_cast<uintptr_t>(15);
+    const uintptr_t end = a + static_cast<uintptr_t>(nw) * sizeof(W);
+#pragma unroll
+    for (int v = 0; v < kWinPieces<W, WC>; ++v) {
+      const uintptr_t pa = a0 + 16u * v;
+      uint32_t n = 0;
+      if (valid && pa < end) n = act_end - pa < 16 ? static_cast<uint32_t>(act_end - pa) : 16u;
+      ptx::cp_async_16(dst + 16 * v, n ? reinterpret_cast<const void *>(pa) : static_cast<const void *>(act), n);
+    }
+    return static_cast<int>((a - a0) >> 2);
   }
 };
 
@@ -1187,8 +1250,12 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         g.oh = static_cast<int>(tq - nq * args.fd_ho.d);
         g.n = static_cast<int>(nq);
       };
-      constexpr uint32_t kSlotBytes = BM * St::kRowBytes;
-      const uint32_t slot0 = ptx::smem_addr(sG) + grp * (kGatherDepth * kSlotBytes) + (t % BM) * St::kRowBytes;
+      const uint32_t g_row = static_cast<uint32_t>(args.g_row);  // staging row pitch
+      const uint32_t kSlotBytes = BM * g_row;
+      const uint32_t slot0 = ptx::smem_addr(sG) + grp * (kGatherDepth * kSlotBytes) + (t % BM) * g_row;
+      const bool win = args.gather_win != 0;
+      const uintptr_t act_end = reinterpret_cast<uintptr_t>(args.act) + static_cast<uintptr_t>(args.act_bytes);
+      uint32_t o4s = 0;  // window offsets of the kGatherDepth slots, 2 bits each
       // issue side: this group's item (itile, ic), kGatherDepth ahead of the consume side
       long long itile = first_tile;
       int ic = 0;
@@ -1202,7 +1269,12 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       if (itile < total_tiles) set_tile(itile);
       auto issue_next = [&](int slot) {
         if (itile < total_tiles) {
-          g.issue(ic, slot0 + slot * kSlotBytes);
+          if (win) {
+            const int o4 = g.issue_win(ic, slot0 + slot * kSlotBytes, act_end);
+            o4s = (o4s & ~(3u << (2 * slot))) | (static_cast<uint32_t>(o4) << (2 * slot));
+          } else {
+            g.issue(ic, slot0 + slot * kSlotBytes);
+          }
           const long long prev = itile;
           step();
           if (kItemStep == 2) step();
@@ -1217,7 +1289,14 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       for (long long k = HV == 2 ? 0 : grp; k < items; k += kItemStep) {
         ptx::cp_async_wait<kGatherDepth - 1>();
         W cur[WC];
-        load_staged<W, WC>(sG + grp * (kGatherDepth * kSlotBytes) + slot * kSlotBytes + (t % BM) * St::kRowBytes, cur);
+        const uint8_t *srow = sG + grp * (kGatherDepth * kSlotBytes) + slot * kSlotBytes + (t % BM) * g_row;
+        if (win) {
+          const int chunk = static_cast<int>(k % nchunks);
+          const int nw = args.words_total - chunk * WC < WC ? args.words_total - chunk * WC : WC;
+          load_window<W, WC>(srow, static_cast<int>((o4s >> (2 * slot)) & 3u), nw, cur);
+        } else {
+          load_staged<W, WC>(srow, cur);
+        }
         const int sa = static_cast<int>(k % NO);
         const long long round = k / NO;
         if (round > 0 && !wait_lane0(opempty(sa), static_cast<uint32_t>((round - 1) & 1))) {
