@@ -221,11 +221,11 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
   const int srow = (chunk_bytes + 15) / 16 * 16;  // Staging::kRowBytes
   const int vec = chunk_bytes % 16 == 0 ? 16 : (chunk_bytes % 8 == 0 ? 8 : wb);
   p.gather_vec = (p.wpr % p.WC == 0) && ((static_cast<long long>(p.wpr) * wb) % vec == 0) ? 1 : 0;
-  // A 1x1 layer whose chunks are not whole aligned vectors copies each
+  // A 1x1 layer whose chunks are not whole 16-byte vectors copies each
   // chunk through the 16-byte-aligned window around it: one more 16-byte
   // piece than the chunk, and an odd number of pieces per staging row, so
   // that a quarter-warp's 16-byte accesses to eight rows hit distinct banks.
-  p.gather_win = (!p.gather_vec && d->R == 1 && d->S == 1) ? 1 : 0;
+  p.gather_win = (!(p.gather_vec && vec == 16) && d->R == 1 && d->S == 1) ? 1 : 0;
   int win_pieces = srow / 16 + 1;
   if (win_pieces % 2 == 0) ++win_pieces;
   const int grow = p.gather_win ? win_pieces * 16 : srow;

@@ -716,6 +716,10 @@ __device__ __forceinline__ void epilogue_row_period(const ConvArgs &args, uint32
   const int nvalid = args.K - ch0 < args.NBc ? args.K - ch0 : args.NBc;
   const float scale = args.out_scale;
   uint32_t *dst = static_cast<uint32_t *>(args.packed_out) + (m * args.out_wpr + ch0 / L);
+  // The last 32-column group may run past the block's channels: its lanes
+  // read the biased zero, and words that lie wholly past the last channel
+  // belong to the next row, so only the block's words are stored.
+  int wleft = (nvalid + L - 1) / L;
   for (int c0 = 0; c0 < nvalid; c0 += 32 * G) {
     uint32_t cur = 0;
     bool open = false;
@@ -736,14 +740,15 @@ __device__ __forceinline__ void epilogue_row_period(const ConvArgs &args, uint32
         cur |= (static_cast<uint32_t>(t) & omask) << (l * OB);
         open = true;
         if (l == L - 1) {
-          if (row_valid) *dst = cur;
+          if (row_valid && wleft > 0) *dst = cur;
           ++dst;
+          --wleft;
           cur = 0;
           open = false;
         }
       }
     }
-    if (open && row_valid) *dst = cur;  // the row's last, partial word
+    if (open && row_valid && wleft > 0) *dst = cur;  // the row's last, partial word
   }
 }
 

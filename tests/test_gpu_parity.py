@@ -257,3 +257,56 @@ def test_bounded_wait_timeout_is_recorded_and_the_context_survives(samd_lib):
     with pytest.raises(samd.SamdError) as e:
         samd.samd_selftest_wait_timeout(10)
     assert e.value.status == samd.SAMD_EINVAL
+
+
+# 1x1 layers whose packed pixel rows are not 16-byte multiples take the
+# gather through 16-byte windows: rows at every 4-byte offset, the last chunk
+# of a pixel running past its words, stride 2, 64-bit words, and the last
+# pixel's window reaching past the end of the activation tensor.
+WINDOW_CASES = [
+    (samd.ConvShape(2, 64, 7, 9, 48, R=1, S=1, pad=0), 6, False, 2, True, 32),    # 52-byte rows (full chunk)
+    (samd.ConvShape(2, 128, 5, 7, 40, R=1, S=1, pad=0), 6, False, 2, True, 32),   # 104-byte rows
+    (samd.ConvShape(1, 192, 9, 5, 24, R=1, S=1, pad=0), 6, True, 5, True, 32),    # 156-byte rows
+    (samd.ConvShape(1, 512, 4, 5, 72, R=1, S=1, pad=0), 6, False, 2, True, 32),   # 412-byte rows, 9 chunks
+    (samd.ConvShape(3, 40, 6, 6, 16, R=1, S=1, pad=0), 4, False, 4, True, 32),    # 20-byte rows, e4m3
+    (samd.ConvShape(2, 30, 5, 5, 20, R=1, S=1, pad=0), 6, False, 3, True, 64),    # 24-byte rows, 64-bit words
+    (samd.ConvShape(2, 128, 9, 9, 40, R=1, S=1, pad=0, stride=2), 6, False, 2, True, 32),  # projection
+]
+
+
+@pytest.mark.parametrize("shape,ba,sa,bw,sw,word_bits", WINDOW_CASES,
+                         ids=lambda v: f"{v.N}x{v.C}x{v.H}x{v.W}-K{v.K}s{v.stride}" if isinstance(v, samd.ConvShape) else None)
+def test_conv_1x1_window_gather(samd_lib, shape, ba, sa, bw, sw, word_bits):
+    assert conv_supported(shape, ba, sa, bw, sw)
+    run_conv_check(shape, ba, sa, bw, sw, word_bits=word_bits, fo_t=(ba, sa, 0, word_bits),
+                   seed=synth.seed_for("win", shape, ba, sa, bw, sw, word_bits))
+
+
+# Packed-only outputs (no int32 accumulator requested) take the fast
+# requantize-and-pack epilogues. Channel counts that are not multiples of 32
+# leave the last 32-column group partly past the last channel: the words the
+# row holds must be exact and nothing past them written (guard words after
+# the output and the neighbouring rows' words stay as they were).
+PACKED_ONLY_K = (40, 70, 290)
+
+
+@pytest.mark.parametrize("fo_signed", SIGNS)
+@pytest.mark.parametrize("fo_bits", BITS)
+def test_conv_packed_only_outputs_partial_groups(samd_lib, fo_bits, fo_signed):
+    for K, (R, word_bits, spacer) in itertools.product(PACKED_ONLY_K, [(3, 32, 0), (1, 32, 0), (3, 64, 0), (1, 32, 1)]):
+        shape = samd.ConvShape(2, 24, 6, 5, K, R=R, S=R, pad=R // 2)
+        a_v, w_v, a_w, w_w, fa, fw = conv_case(shape, 4, False, 3, True,
+                                               synth.seed_for("po", K, R, fo_bits, fo_signed, word_bits))
+        fo = samd.fmt(fo_bits, fo_signed, spacer, word_bits)
+        shift = harness_shift(4, 3, fo_bits, shape.C * shape.R * shape.S)
+        n = samd.samd_packed_words(fo, shape.N * shape.Ho * shape.Wo, K)
+        guard = 64
+        buf = torch.full((n + guard,), 0x5A5A5A5A, dtype=samd.word_dtype(fo), device="cuda")
+        ws = samd.conv_workspace(shape, fa, fw)
+        samd.samd_conv2d(shape.desc(), fa, a_w, fw, w_w, None, fo, buf, shift, ws)
+        torch.cuda.synchronize()
+        got = np_words(buf, word_bits)
+        want = oracle_requant_pack(oracle_conv_nhwc(a_v, w_v, shape), shift, fo)
+        assert np.array_equal(got[:n], want), (K, R, word_bits, spacer)
+        assert np.array_equal(got[n:], np_words(torch.full((guard,), 0x5A5A5A5A, dtype=samd.word_dtype(fo)), word_bits))
+    assert_status_clean()
