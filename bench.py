@@ -151,13 +151,14 @@ class ClockSampler:
 
 # ---- CPU oracle baseline ---------------------------------------------------------------
 
-def cpu_oracle_rate(layers, seconds: float):
-    """The oracle's direct convolution on one image of each layer in turn,
-    all host cores, until `seconds` have passed. Returns (MAC/s, threads, sample)."""
+def cpu_oracle_rate(layers, seconds: float, threads: int = 0):
+    """The oracle's direct convolution on one image of each layer in turn, on
+    `threads` host threads (0: all cores), until `seconds` have passed.
+    Returns (MAC/s, threads, sample)."""
     import oracle
     from paper_1809_10572_gb300 import synth
 
-    threads = os.cpu_count() or 1
+    threads = threads or os.cpu_count() or 1
     done_macs, t0, k = 0, time.perf_counter(), 0
     names = []
     while time.perf_counter() - t0 < seconds or k == 0:
@@ -545,7 +546,9 @@ def run_samd(args, layers):
     line["clocks"] = clk
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         v, cores, sample = cpu_oracle_rate(layers, args.cpu_seconds)
-        line["cpu_baseline"] = {"value": v, "unit": "MAC/s", "cores": cores, "kind": "oracle", "sample": sample}
+        v1, _, sample1 = cpu_oracle_rate(layers, args.cpu_seconds / 3, threads=1)
+        line["cpu_baseline"] = {"value": v, "unit": "MAC/s", "cores": cores, "kind": "oracle", "sample": sample,
+                                "value_1thread": v1, "sample_1thread": sample1}
     if rank == 0:
         print(json.dumps(line), flush=True)
     d.close()
