@@ -930,14 +930,19 @@ __device__ __forceinline__ void issue_taps(uint32_t d, uint32_t dn, uint64_t a, 
 //               needs are gathered with cp.async and widened once into one of
 //               two halo buffers; every tap reads the halo through a
 //               descriptor shifted by r * row_step + s rows.
-//               GATHER: two groups of four warps take alternate (tile, chunk)
-//               items; each thread gathers its pixel's packed words (implicit
+//               GATHER: each thread gathers its pixel's packed words (implicit
 //               im2col, zero padding) through a cp.async ring and widens them
-//               into a ring of A tiles.
+//               into a ring of A tiles; with HV = 1 two groups of four warps
+//               take alternate (tile, chunk) items, with HV = 2 the two groups
+//               fill the two halves of every item. 1x1 layers whose pixel
+//               rows are not 16-byte multiples copy 16-byte windows.
 //   warps 10-17 epilogue: tcgen05.ld, exact integers, optional int32 store,
-//               optional requantize-and-pack. Warps 10-13 drain accumulator 0
-//               (the CTA's even tiles), warps 14-17 accumulator 1; warp w
-//               reads the TMEM lanes of quadrant w % 4.
+//               optional requantize-and-pack. HV = 1: warps 10-13 drain
+//               accumulator 0 (the CTA's even tiles), warps 14-17
+//               accumulator 1; HV = 2: warps 10-13 drain the first half and
+//               14-17 the second half of every tile. Warp w reads the TMEM
+//               lanes of quadrant w % 4. A first, store-free pass over the
+//               first tile fetches the epilogue's code early.
 // Every wait is bounded; a role that gives up records SAMD_ETIMEOUT and stops.
 template <typename W, int BITS, bool SIGNED, bool HALO, bool FP8, bool FULL, int HV>
 __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant__ CUtensorMap tmap_b,
@@ -1016,7 +1021,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         // the CTA does not exit with a copy in flight, whatever the other roles do
         for (int c = 0; c < nchunks; ++c) ptx::mbar_wait_bounded(full_b(c), 0, &quiet, kWaitLimitNs);
       } else {
-        long long cb = 0, issued_from = 0;
+        long long cb = 0;
         for (long long tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
           const int nb = static_cast<int>(tile / args.grid_m);
           for (int c = 0; c < nchunks; ++c, ++cb) {
@@ -1032,7 +1037,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
           }
         }
         if (!ok) {  // leave no copy in flight: wait (bounded) for the last ring's worth
-          for (long long k = (cb - STB > issued_from ? cb - STB : issued_from); k < cb; ++k)
+          for (long long k = (cb > STB ? cb - STB : 0); k < cb; ++k)
             ptx::mbar_wait_bounded(full_b(static_cast<int>(k % STB)), static_cast<uint32_t>((k / STB) & 1), &quiet,
                                    kWaitLimitNs / 10);
         }
