@@ -56,6 +56,9 @@ def parse_args():
                          "total (rotate), or by flushing L2 before every step (flush)")
     ap.add_argument("--streams", type=int, default=8,
                     help="independent layers of a step run on this many streams (graph branches)")
+    ap.add_argument("--connections", type=int, default=0,
+                    help="CUDA_DEVICE_MAX_CONNECTIONS for this process (hardware work queues the streams map "
+                         "onto; 0: leave the environment as it is)")
     return ap.parse_args()
 
 
@@ -236,7 +239,8 @@ def workload_config(args, layers):
                    if args.l2 == "rotate" else
                    "flushed before every step (512 MiB write, then 512 MiB read); inputs resident in HBM"),
             "weights": "prepared once into the tensor-core operand layout (samd_conv2d_prepare), not in the step",
-            "launch": f"one CUDA graph per step; independent layers fanned out over {args.streams} streams; "
+            "launch": f"one CUDA graph per step; independent layers fanned out over {args.streams} streams"
+                      f"{f' ({args.connections} hardware work queues)' if args.connections else ''}; "
                       f"each CTA at least {args.tiles_per_cta or (8 if args.workload == 'sweep' else 4)} reference tiles "
                       f"of work (samd_conv2d_set_min_tiles_per_cta)",
             "parallelism": f"replicas x{args.gpus}"}
@@ -351,13 +355,12 @@ def measured_traffic(args):
     if rec.get("csrc_sha256") != csrc_digest():
         return None, "kernel sources changed since the ncu traffic capture"
     return rec["dram_bytes_per_launch"], ("ncu dram__bytes_read.sum + dram__bytes_write.sum, mean over the step's "
-                                          f"{rec['launches']} launches (profiles/conv_kernel_sweep_traffic.md)")
+                                          f"{rec['launches']} launches")
 
 
 def run_samd(args, layers):
     import torch
 
-    import oracle  # noqa: F401  (CPU-baseline leg only)
     from paper_1809_10572_gb300 import samd, workloads
 
     ws, rank, local = dist_env()
@@ -491,10 +494,19 @@ def run_samd(args, layers):
     peak_src = "measured" if bf16_peak else "fallback"
     bf16_peak = bf16_peak or 1900.0
     # The peak of each layer is that of its operand type: fp16 runs at the
-    # bf16 rate; e4m3 at twice it (the nominal 4.5 / 2.25 PFLOP/s dense
-    # ratio). The step's peak is the rate at which every layer would run at
-    # its own peak: 2 x step MACs / sum of the layers' ideal times.
-    ideal_s = sum(2.0 * b["layer"].macs / ((2.0 if b["operand_bits"] == 8 else 1.0) * bf16_peak * 1e12) for b in built)
+    # bf16 rate (MEASURED_PEAKS.json, burst); e4m3 at the e4m3 rate measured
+    # here (cuBLASLt through torch._scaled_mm), or at twice the bf16 rate (the
+    # nominal 4.5 / 2.25 PFLOP/s dense ratio) if that cannot be measured. The
+    # step's peak is the rate at which every layer would run at its own peak:
+    # 2 x step MACs / sum of the layers' ideal times.
+    e4m3 = measure_e4m3_peak(dev)
+    e4m3_peak = e4m3["tflops"] or 2.0 * bf16_peak
+    e4m3_src = "measured (torch._scaled_mm 8192^3)" if e4m3["tflops"] else f"2 x {peak_src} bf16"
+
+    def layer_peak(b):
+        return e4m3_peak if b["operand_bits"] == 8 else bf16_peak
+
+    ideal_s = sum(2.0 * b["layer"].macs / (layer_peak(b) * 1e12) for b in built)
     step_peak = 2.0 * step_macs / ideal_s / 1e12
     n_e4m3 = sum(1 for b in built if b["operand_bits"] == 8)
     achieved_tflops = 2.0 * step_macs / (ms_per_step * 1e-3) / 1e12
@@ -502,9 +514,14 @@ def run_samd(args, layers):
     roofline = {"kernel": "conv_kernel", "bound": "tensor", "achieved": achieved_tflops, "peak": step_peak,
                 "unit": "TFLOP/s", "frac": achieved_tflops / step_peak, "traffic": traffic,
                 "traffic_note": traffic_note,
-                "peak_source": f"{peak_src} bf16 burst {bf16_peak:.1f} TFLOP/s for fp16 layers, x2 for e4m3 layers "
-                               f"({n_e4m3} of {len(built)} layers), MAC-weighted",
-                "note": "achieved = 2 x direct-conv MACs of the step / step time (all launches are the conv kernel)"}
+                "peak_source": f"fp16 layers: {peak_src} bf16 burst {bf16_peak:.1f} TFLOP/s; e4m3 layers "
+                               f"({n_e4m3} of {len(built)}): {e4m3_src} {e4m3_peak:.1f} TFLOP/s; MAC-weighted",
+                "e4m3_peak": e4m3,
+                "frac_vs_nominal_ratio": achieved_tflops / (2.0 * step_macs / sum(
+                    2.0 * b["layer"].macs / ((2.0 if b["operand_bits"] == 8 else 1.0) * bf16_peak * 1e12)
+                    for b in built) / 1e12),
+                "note": "achieved = 2 x direct-conv MACs of the step / step time (all launches are the conv kernel); "
+                        "frac_vs_nominal_ratio takes e4m3 at 2 x the bf16 peak instead"}
 
     line = {
         "metric": METRIC, "value": value, "unit": "MAC/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
@@ -555,27 +572,83 @@ def run_samd(args, layers):
     return 0
 
 
-def measure_int8_peak(dev):
+def _best_time(fn, reps=5):
     import torch
 
+    fn()
+    torch.cuda.synchronize()
+    best = None
+    for _ in range(reps):
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record()
+        fn()
+        s1.record()
+        s1.synchronize()
+        t = s0.elapsed_time(s1) * 1e-3
+        best = t if best is None else min(best, t)
+    return best
+
+
+def measure_int8_peak(dev):
+    """Dense int8 tensor-core rate, the best of torch._int_mm (cuBLASLt) on
+    8192^3 and the hand-written mma.sync m16n8k32 s8 loop (libsamd_peaks)."""
+    import ctypes
+
+    import torch
+
+    from paper_1809_10572_gb300 import build as samd_build
+
+    res = {}
     try:
         n = 8192
         a = torch.randint(-128, 127, (n, n), dtype=torch.int8, device=dev)
         b = torch.randint(-128, 127, (n, n), dtype=torch.int8, device=dev)
-        torch._int_mm(a, b)
-        torch.cuda.synchronize()
-        best = None
-        for _ in range(5):
-            s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            s0.record()
-            torch._int_mm(a, b)
-            s1.record()
-            s1.synchronize()
-            t = s0.elapsed_time(s1) * 1e-3
-            best = t if best is None else min(best, t)
-        return {"tops": 2 * n ** 3 / best / 1e12, "how": "torch._int_mm int8 8192^3, best of 5"}
+        res["int_mm_tops"] = 2 * n ** 3 / _best_time(lambda: torch._int_mm(a, b)) / 1e12
+        del a, b
     except Exception as e:  # noqa: BLE001
-        return {"tops": None, "how": f"torch._int_mm unavailable: {type(e).__name__}"}
+        res["int_mm_tops"] = None
+        res["int_mm_error"] = type(e).__name__
+    try:
+        lib = ctypes.CDLL(samd_build.build_peaks())
+        lib.samd_peak_imma_s8.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+                                          ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_double)]
+        lib.samd_peak_imma_s8.restype = ctypes.c_int
+        scratch = torch.zeros(4, dtype=torch.int32, device=dev)
+        sms = torch.cuda.get_device_properties(dev).multi_processor_count
+        best = None
+        for per_sm in (2, 4, 8):
+            ms, macs = ctypes.c_float(0), ctypes.c_double(0)
+            rc = lib.samd_peak_imma_s8(sms * per_sm, 4096, scratch.data_ptr(), ctypes.byref(ms), ctypes.byref(macs))
+            if rc == 0 and ms.value > 0:
+                tops = 2 * macs.value / (ms.value * 1e-3) / 1e12
+                best = tops if best is None else max(best, tops)
+        res["mma_sync_s8_tops"] = best
+    except Exception as e:  # noqa: BLE001
+        res["mma_sync_s8_tops"] = None
+        res["mma_sync_error"] = f"{type(e).__name__}: {e}"
+    vals = [v for v in (res.get("int_mm_tops"), res.get("mma_sync_s8_tops")) if v]
+    res["tops"] = max(vals) if vals else None
+    res["how"] = ("best of torch._int_mm int8 8192^3 (best of 5) and a hand-written mma.sync m16n8k32 s8 loop on "
+                  "register operands (2, 4, 8 blocks of 256 threads per SM, 4096 x 8 MMAs per warp)")
+    return res
+
+
+def measure_e4m3_peak(dev):
+    """Dense e4m3 tensor-core rate: torch._scaled_mm (cuBLASLt) on 8192^3 with
+    unit scales and fp32... bf16 output, best of 5 -- the peak of the
+    convolution's e4m3 layers."""
+    import torch
+
+    try:
+        n = 8192
+        a = torch.randn(n, n, device=dev).to(torch.float8_e4m3fn)
+        b = torch.randn(n, n, device=dev).to(torch.float8_e4m3fn).t()
+        one = torch.ones((), device=dev)
+        t = _best_time(lambda: torch._scaled_mm(a, b, scale_a=one, scale_b=one, out_dtype=torch.bfloat16))
+        return {"tflops": 2 * n ** 3 / t / 1e12,
+                "how": "torch._scaled_mm e4m3 x e4m3 -> bf16, 8192^3, unit scales, best of 5"}
+    except Exception as e:  # noqa: BLE001
+        return {"tflops": None, "how": f"torch._scaled_mm unavailable: {type(e).__name__}: {e}"}
 
 
 def measure_e2e(built, step_macs, args, dev, ws, d):
@@ -651,6 +724,8 @@ def measure_e2e(built, step_macs, args, dev, ws, d):
 
 def main():
     args = parse_args()
+    if args.connections:  # read by the CUDA runtime when it creates the context, so set before any CUDA call
+        os.environ["CUDA_DEVICE_MAX_CONNECTIONS"] = str(args.connections)
     from paper_1809_10572_gb300 import workloads
 
     layers = workloads.WORKLOADS[args.workload]()

@@ -221,11 +221,15 @@ SAMD_API samd_status samd_conv2d_prepared(const samd_conv_desc *desc, samd_fmt f
  * convenience. Same arguments and results as samd_conv2d, without the
  * workspace: the widened weights go to a static device array of
  * 8 MiB (8388608 bytes) inside the library, held on every GPU that loads it
- * until the process exits. A layer whose widened weights need more
- * (samd_conv2d_workspace_size > 8 MiB, e.g. 3x3 convolutions with far more
- * than 512 x 512 channels) is rejected with SAMD_EUNSUP before any launch.
- * The first call on a device looks the array's device address up (once per
- * device, with that device current); make that first call before capturing
+ * until the process exits. A call whose widened weights -- for its own desc,
+ * fa, fw and output format fo -- need more than 8 MiB (e.g. 3x3
+ * convolutions with far more than 512 x 512 channels) is rejected with
+ * SAMD_EUNSUP before any launch; samd_conv2d_workspace_size, the largest
+ * size over every output format, bounds that need from above, so a layer
+ * with samd_conv2d_workspace_size <= 8 MiB is always accepted.
+ * The first call in a CUDA context looks the array's device address up
+ * (once per context, with that context current; a context created after
+ * cudaDeviceReset looks it up again); make that first call before capturing
  * a stream into a CUDA graph. Every call reuses the same array and rewrites
  * the part it reads before reading it, so no earlier contents leak into a
  * result; but calls whose work overlaps on the GPU (different streams, no

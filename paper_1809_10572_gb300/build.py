@@ -3,8 +3,10 @@
 Each .cu translation unit under csrc/ is compiled in parallel with nvcc
 (-gencode arch=compute_103a,code=sm_103a) -- conv_inst.cu once per kernel
 instantiation group -- and the objects are linked into
-paper_1809_10572_gb300/lib/libsamd.so. A rebuild happens only when a source
-or header is newer than the library.
+paper_1809_10572_gb300/lib/libsamd.so. The measurement kernels under peaks/
+(tensor-core rate microbenchmarks, not part of the hot path) go into
+lib/libsamd_peaks.so. A rebuild happens only when a source or header is
+newer than the library.
 """
 from __future__ import annotations
 
@@ -20,6 +22,8 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 LIBDIR = os.path.join(PKG, "lib")
 LIB = os.path.join(LIBDIR, "libsamd.so")
+PEAKS_DIR = os.path.join(PKG, "peaks")
+PEAKS_LIB = os.path.join(LIBDIR, "libsamd_peaks.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
               "-Xcompiler", "-fvisibility=hidden", "-I", os.path.join(ROOT, "include")]
@@ -63,7 +67,30 @@ def up_to_date() -> bool:
     return all(os.path.getmtime(p) <= t for p in _inputs())
 
 
+def peaks_up_to_date() -> bool:
+    if not os.path.exists(PEAKS_LIB):
+        return False
+    t = os.path.getmtime(PEAKS_LIB)
+    return all(os.path.getmtime(p) <= t for p in glob.glob(os.path.join(PEAKS_DIR, "*.cu")))
+
+
+def build_peaks(force: bool = False) -> str:
+    """lib/libsamd_peaks.so from peaks/*.cu (one nvcc call)."""
+    if not force and peaks_up_to_date():
+        return PEAKS_LIB
+    os.makedirs(LIBDIR, exist_ok=True)
+    srcs = sorted(glob.glob(os.path.join(PEAKS_DIR, "*.cu")))
+    tmp = PEAKS_LIB + ".tmp"
+    cmd = [nvcc()] + ARCH + NVCC_FLAGS + ["-shared", "-o", tmp] + srcs
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    if r.returncode != 0:
+        raise RuntimeError(f"nvcc failed on peaks/:\n{r.stderr}")
+    os.replace(tmp, PEAKS_LIB)
+    return PEAKS_LIB
+
+
 def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | None = None) -> str:
+    build_peaks(force)
     if not force and up_to_date():
         return LIB
     os.makedirs(LIBDIR, exist_ok=True)

@@ -22,22 +22,63 @@ __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
 
 namespace conv {
 
-// cudaFuncSetAttribute once per (kernel, device), so that launches made
+// Identity of the current CUDA context (cuCtxGetId), unique for the life of
+// the process: a cache entry made for one context is never taken for a
+// context created later, such as the primary context a device gets again
+// after cudaDeviceReset (which reloads the module: kernel attributes and
+// symbol addresses change). If the runtime has not made a context current
+// yet, cudaSetDevice makes the device's primary context current (no
+// allocation).
+cudaError_t current_context_id(unsigned long long *id) {
+  using GetCurrentFn = CUresult (*)(CUcontext *);
+  using GetIdFn = CUresult (*)(CUcontext, unsigned long long *);
+  static GetCurrentFn get_current = nullptr;
+  static GetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<GetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<GetIdFn>(p);
+  });
+  if (!get_current || !get_id) return cudaErrorNotSupported;
+  CUcontext ctx = nullptr;
+  if (get_current(&ctx) != CUDA_SUCCESS) return cudaErrorDeviceUninitialized;
+  if (!ctx) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaSetDevice(dev);
+    if (e != cudaSuccess) return e;
+    if (get_current(&ctx) != CUDA_SUCCESS || !ctx) return cudaErrorDeviceUninitialized;
+  }
+  return get_id(ctx, id) == CUDA_SUCCESS ? cudaSuccess : cudaErrorDeviceUninitialized;
+}
+
+// cudaFuncSetAttribute once per (kernel, context), so that launches made
 // while a stream is being captured into a graph issue no other CUDA call.
 // The dynamic limit is the per-block maximum minus the kernel's static
 // shared memory. Returns cudaErrorInvalidValue if `smem` does not fit.
 cudaError_t ensure_smem_attr(const void *kern, size_t smem) {
+  constexpr int kSlots = 512;
   static std::mutex mu;
-  static const void *done_fn[512];
-  static int done_dev[512];
-  static size_t done_smem[512];
-  static int n_done = 0;
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  static const void *done_fn[kSlots];
+  static unsigned long long done_ctx[kSlots];
+  static size_t done_smem[kSlots];
+  static int n_done = 0, next_slot = 0;
+  unsigned long long ctx = 0;
+  cudaError_t e = current_context_id(&ctx);
   if (e != cudaSuccess) return e;
   std::lock_guard<std::mutex> lock(mu);
   for (int i = 0; i < n_done; ++i)
-    if (done_fn[i] == kern && done_dev[i] == dev) return smem <= done_smem[i] ? cudaSuccess : cudaErrorInvalidValue;
+    if (done_fn[i] == kern && done_ctx[i] == ctx) return smem <= done_smem[i] ? cudaSuccess : cudaErrorInvalidValue;
+  int dev = 0;
+  e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
   int optin = 0;
   e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
   if (e != cudaSuccess) return e;
@@ -47,12 +88,11 @@ cudaError_t ensure_smem_attr(const void *kern, size_t smem) {
   const size_t limit = static_cast<size_t>(optin) - fa.sharedSizeBytes;
   e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(limit));
   if (e != cudaSuccess) return e;
-  if (n_done < 512) {
-    done_fn[n_done] = kern;
-    done_dev[n_done] = dev;
-    done_smem[n_done] = limit;
-    ++n_done;
-  }
+  const int slot = n_done < kSlots ? n_done++ : next_slot;  // when full, entries are replaced in turn
+  if (n_done == kSlots) next_slot = (slot + 1) % kSlots;
+  done_fn[slot] = kern;
+  done_ctx[slot] = ctx;
+  done_smem[slot] = limit;
   return smem <= limit ? cudaSuccess : cudaErrorInvalidValue;
 }
 
@@ -365,24 +405,33 @@ bool layout_ok(const Plan &p) {
          (p.hv == 1 || p.hv == 2);
 }
 
-// Device address of a __device__ symbol on the current device, looked up
-// once per device (the symbol's host-side name is not a device address).
+// Device address of a __device__ symbol in the current context, looked up
+// once per context (the symbol's host-side name is not a device address; a
+// context made after a device reset loads the module again, at a new address).
 struct SymbolAddr {
+  static constexpr int kSlots = 64;
   std::mutex mu;
-  void *ptr[64] = {nullptr};
+  unsigned long long ctx[kSlots] = {0};
+  void *ptr[kSlots] = {nullptr};
+  int n = 0, next = 0;
   cudaError_t get(const void *symbol, void **out) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
+    unsigned long long id = 0;
+    cudaError_t e = current_context_id(&id);
     if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
     std::lock_guard<std::mutex> lock(mu);
-    if (!ptr[dev]) {
-      void *p = nullptr;
-      e = cudaGetSymbolAddress(&p, symbol);
-      if (e != cudaSuccess) return e;
-      ptr[dev] = p;
-    }
-    *out = ptr[dev];
+    for (int i = 0; i < n; ++i)
+      if (ctx[i] == id) {
+        *out = ptr[i];
+        return cudaSuccess;
+      }
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, symbol);
+    if (e != cudaSuccess) return e;
+    const int slot = n < kSlots ? n++ : next;  // when full, entries are replaced in turn
+    if (n == kSlots) next = (slot + 1) % kSlots;
+    ctx[slot] = id;
+    ptr[slot] = p;
+    *out = p;
     return cudaSuccess;
   }
 };
@@ -621,7 +670,8 @@ samd_status conv2d_nhwc_noalloc(const samd_conv_desc *d, samd_fmt fa, const void
   conv::Plan p;
   samd_status st = conv::make_plan(d, fa, fw, packed_out ? fo : conv::none_fmt(), p);
   if (st != SAMD_OK) return st;
-  if (p.ws_bytes > kNoallocScratchBytes) return SAMD_EUNSUP;  // the layer's weights do not fit the static scratch
+  // the widened weights of this call (shape, formats, output format) must fit
+  if (p.ws_bytes > kNoallocScratchBytes) return SAMD_EUNSUP;
   void *scratch = nullptr;
   if (conv::g_scratch_addr.get(reinterpret_cast<const void *>(&g_noalloc_scratch), &scratch) != cudaSuccess)
     return SAMD_ECUDA;

@@ -9,9 +9,15 @@
 // lane-by-lane loop would run 16-32 iterations per word. Words move with
 // 128-bit loads and stores.
 //
-// Everything else (spacer bits, saturating multiply of wide lanes,
-// requantize into another format) takes the per-lane path: one thread per
-// output word, bit-field extract, integer op, clamp or wrap, insert.
+// Formats with permanent spacer bits (section 2.1, Fig. 2) and the same
+// input and output format take word-level forms too: the zero spacer bits
+// above each lane catch the carry of an add and the borrow of a subtract, so
+// a wrapping add is one add and one mask, and the saturating forms read each
+// lane's carry or borrow from its first spacer bit; the other ops use the
+// temporary-spacer forms with masks over the spacer-separated fields.
+//
+// Requantize into another format takes the per-lane path: one thread per
+// output word, bit-field extract, integer op, clamp, insert.
 #include "samd_internal.cuh"
 
 namespace samd {
@@ -253,6 +259,159 @@ __global__ void __launch_bounds__(kThreads)
   }
 }
 
+// ---- formats with permanent spacer bits ------------------------------------
+//
+// A lane field is bits data bits plus spacer zero bits above them, L fields
+// per word (FieldMasks, samd_internal.cuh).
+
+template <typename W>
+__device__ __forceinline__ W field_relu(W a, const FieldMasks<W> &f, bool is_signed) {
+  if (!is_signed) return a;
+  return a & ~spread_down<W>(a & f.msb, f.bits - 1);
+}
+
+template <typename W>
+__device__ __forceinline__ W field_shift(W a, int shift, W keep, const FieldMasks<W> &f, bool is_signed) {
+  if (shift == 0) return a;
+  W r = (a >> shift) & keep;
+  if (is_signed) {
+    W sg = a & f.msb;
+    W t = sg >> (shift - 1);
+    r |= (sg - t) | sg;  // sign fill of the top `shift` data bits of negative lanes
+  }
+  return r;
+}
+
+// Fig. 2: with the spacers zero (canonical inputs) the word add leaves each
+// lane's carry in its first spacer bit. Wrapping: drop it. Saturating,
+// unsigned: a set carry bit turns the lane's data bits all ones. Signed:
+// overflow where same-sign operands give a result of the other sign.
+template <typename W>
+__device__ __forceinline__ W field_add(W a, W b, const FieldMasks<W> &f, bool is_signed, bool sat) {
+  const W s = a + b;
+  if (!sat) return s & f.live;
+  if (!is_signed) {
+    const W c = s & f.carry;
+    return (s | (c - (c >> f.bits))) & f.live;
+  }
+  const W w = s & f.live;
+  const W E = spread_down<W>(~(a ^ b) & (a ^ w) & f.msb, f.bits - 1);  // overflowed lanes
+  const W na = a & f.msb;                                                 // their operands' sign
+  const W sat_v = (E & ~spread_down<W>(na, f.bits - 1) & ~f.msb & f.live) | (E & na);  // 011..1 or 100..0
+  return (w & ~E) | sat_v;
+}
+
+// (a | carry) - b: each field computes 2^bits + a - b > 0, so no borrow
+// leaves a field, and the carry bit stays set exactly where a >= b
+// (unsigned).
+template <typename W>
+__device__ __forceinline__ W field_sub(W a, W b, const FieldMasks<W> &f, bool is_signed, bool sat) {
+  const W d = (a | f.carry) - b;
+  if (!sat) return d & f.live;
+  if (!is_signed) {
+    const W ge = d & f.carry;
+    return d & (ge - (ge >> f.bits)) & f.live;  // lanes with a < b clamp to 0
+  }
+  const W w = d & f.live;
+  const W E = spread_down<W>((a ^ b) & (a ^ w) & f.msb, f.bits - 1);
+  const W na = a & f.msb;
+  const W sat_v = (E & ~spread_down<W>(na, f.bits - 1) & ~f.msb & f.live) | (E & na);
+  return (w & ~E) | sat_v;
+}
+
+template <typename W>
+__device__ __forceinline__ W field_mul(W a, W b, const FieldMasks<W> &f, bool is_signed, bool sat) {
+  if (!sat && f.bits <= 2) {
+    // Fig. 6 shift-and-add over the fields: step j adds a << j where bit j
+    // of the lane of b is set, cut at the top of the lane's data bits
+    W acc = 0;
+    for (int j = 0; j < f.bits; ++j) {
+      const W bit = b & (f.lsb << j);
+      const W write = (bit << (f.bits - j)) - bit;
+      acc = (acc + ((a << j) & write)) & f.live;  // the spacer catches the carry
+    }
+    return acc;
+  }
+  const uint32_t lm = (1u << f.bits) - 1;
+  const int lo = lane_lo(f.bits, is_signed), hi = lane_hi(f.bits, is_signed);
+  W r = 0;
+  for (int i = 0; i < f.L; ++i) {
+    const uint32_t pa = static_cast<uint32_t>(a >> (i * f.fw)) & lm;
+    const uint32_t pb = static_cast<uint32_t>(b >> (i * f.fw)) & lm;
+    uint32_t p;
+    if (sat)
+      p = static_cast<uint32_t>(clamp_int(lane_value(pa, f.bits, is_signed) * lane_value(pb, f.bits, is_signed), lo,
+                                          hi)) & lm;
+    else
+      p = (pa * pb) & lm;
+    r |= W(p) << (i * f.fw);
+  }
+  return r;
+}
+
+template <typename W, int OP>
+__device__ __forceinline__ W field_op(W a, W b, const FieldMasks<W> &f, bool is_signed, bool sat, int shift,
+                                      W keep) {
+  if constexpr (OP == SAMD_ADD) return field_add<W>(a, b, f, is_signed, sat);
+  else if constexpr (OP == SAMD_SUB) return field_sub<W>(a, b, f, is_signed, sat);
+  else if constexpr (OP == SAMD_MUL) return field_mul<W>(a, b, f, is_signed, sat);
+  else if constexpr (OP == SAMD_RELU) return field_relu<W>(a, f, is_signed);
+  else return field_shift<W>(a, shift, keep, f, is_signed);
+}
+
+template <typename W, int OP>
+__global__ void __launch_bounds__(kThreads)
+    ew_field_kernel(const W *__restrict__ a, const W *__restrict__ b, W *__restrict__ out, int64_t nwords,
+                    const FieldMasks<W> f, int is_signed, int sat, int shift) {
+  constexpr int V = 16 / sizeof(W);
+  constexpr bool kBinary = (OP == SAMD_ADD || OP == SAMD_SUB || OP == SAMD_MUL);
+  W keep = 0;
+  if (OP == SAMD_REQUANT) {
+    const int s = shift < f.bits ? shift : f.bits;
+    keep = f.lsb * ((W(1) << (f.bits - s)) - 1);
+    shift = s;
+  }
+  const int64_t nvec = nwords / V;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < nvec; v += stride) {
+    const uint4 ra = __ldcs(reinterpret_cast<const uint4 *>(a) + v);
+    uint4 rb = ra;
+    if (kBinary) rb = __ldcs(reinterpret_cast<const uint4 *>(b) + v);
+    W wa[V], wb[V], wo[V];
+    memcpy(wa, &ra, 16);
+    memcpy(wb, &rb, 16);
+#pragma unroll
+    for (int k = 0; k < V; ++k) wo[k] = field_op<W, OP>(wa[k], wb[k], f, is_signed, sat, shift, keep);
+    uint4 ro;
+    memcpy(&ro, wo, 16);
+    __stcs(reinterpret_cast<uint4 *>(out) + v, ro);
+  }
+  for (int64_t w = nvec * V + blockIdx.x * (int64_t)blockDim.x + threadIdx.x; w < nwords; w += stride) {
+    const W x = a[w];
+    const W y = kBinary ? b[w] : x;
+    out[w] = field_op<W, OP>(x, y, f, is_signed, sat, shift, keep);
+  }
+}
+
+template <typename W>
+cudaError_t field_dispatch(samd_op op, samd_fmt f, const void *a, const void *b, void *out, int64_t n, int shift,
+                           int sat, cudaStream_t s) {
+  const int64_t nwords = words_per_row(f, n);
+  const int grid = grid_for(nwords / (16 / sizeof(W)) + 1, kThreads, sm_count() * 8);
+  const FieldMasks<W> m = field_masks<W>(f);
+  const W *pa = static_cast<const W *>(a);
+  const W *pb = static_cast<const W *>(b);
+  W *po = static_cast<W *>(out);
+  switch (op) {
+    case SAMD_ADD: ew_field_kernel<W, SAMD_ADD><<<grid, kThreads, 0, s>>>(pa, pb, po, nwords, m, f.is_signed, sat, shift); break;
+    case SAMD_SUB: ew_field_kernel<W, SAMD_SUB><<<grid, kThreads, 0, s>>>(pa, pb, po, nwords, m, f.is_signed, sat, shift); break;
+    case SAMD_MUL: ew_field_kernel<W, SAMD_MUL><<<grid, kThreads, 0, s>>>(pa, pb, po, nwords, m, f.is_signed, sat, shift); break;
+    case SAMD_RELU: ew_field_kernel<W, SAMD_RELU><<<grid, kThreads, 0, s>>>(pa, pb, po, nwords, m, f.is_signed, sat, shift); break;
+    default: ew_field_kernel<W, SAMD_REQUANT><<<grid, kThreads, 0, s>>>(pa, pb, po, nwords, m, f.is_signed, sat, shift); break;
+  }
+  return cudaGetLastError();
+}
+
 template <typename W, int OP>
 cudaError_t swar_dispatch_bits(int bits, const void *a, const void *b, void *out, int64_t nwords, int is_signed,
                                int sat, int shift, cudaStream_t s) {
@@ -306,6 +465,10 @@ cudaError_t lane_dispatch(samd_op op, samd_fmt fa, const void *a, const void *b,
 
 cudaError_t launch_elementwise(samd_op op, samd_fmt fa, const void *a, const void *b, samd_fmt fo, void *out,
                                int64_t n, int shift, int saturate, cudaStream_t s) {
+  if (same_fmt(fa, fo) && fa.spacer != 0) {  // permanent spacer bits: the field forms above
+    if (fa.word_bits == 32) return field_dispatch<uint32_t>(op, fa, a, b, out, n, shift, saturate, s);
+    return field_dispatch<uint64_t>(op, fa, a, b, out, n, shift, saturate, s);
+  }
   bool swar = same_fmt(fa, fo) && fa.spacer == 0;
   if (swar) {
     int64_t nwords = words_per_row(fa, n);

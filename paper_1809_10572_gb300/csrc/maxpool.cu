@@ -1,11 +1,12 @@
 // maxpool.cu -- lane-wise 2x2 max-pool, stride 2, on NHWC tensors packed
 // along C (used between the VGG-16 blocks; the paper has no pooling).
 //
-// For spacer-free lanes the max of two words is
-// taken for all lanes at once: a lane-wise subtract with the MSBs as
-// temporary spacers (section 3, Fig. 5) yields each lane's borrow, i.e.
-// a < b, which selects the larger lane. Signed lanes are compared after
-// flipping their sign bits (two's complement order = offset-binary order).
+// The max of two words is taken for all lanes at once. Spacer-free lanes: a
+// lane-wise subtract with the MSBs as temporary spacers (section 3, Fig. 5)
+// yields each lane's borrow, i.e. a < b, which selects the larger lane.
+// Lanes with permanent spacer bits (Fig. 2) read a >= b from the first
+// spacer bit of (a | carry) - b. Signed lanes are compared after flipping
+// their sign bits (two's complement order = offset-binary order).
 #include <cstring>
 
 #include "samd_internal.cuh"
@@ -79,50 +80,37 @@ __global__ void __launch_bounds__(kThreads) maxpool_swar_kernel(const W *__restr
   }
 }
 
+// Formats with permanent spacer bits: the same row walk, one word per
+// (pixel, word) pair, lane-wise max by field_max.
 template <typename W>
-__global__ void __launch_bounds__(kThreads) maxpool_lane_kernel(const W *__restrict__ in, W *__restrict__ out, int N,
-                                                                int H, int W_, int wpr, int bits, int is_signed,
-                                                                int lane_w, int L) {
-  const int Ho = H / 2, Wo = W_ / 2;
-  const int64_t total = (int64_t)N * Ho * Wo * wpr;
-  const uint32_t lm = (1u << bits) - 1;
-  for (int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; t < total; t += (int64_t)gridDim.x * blockDim.x) {
-    int64_t px = t / wpr;
-    int wi = static_cast<int>(t - px * wpr);
-    int j = static_cast<int>(px % Wo);
-    int64_t r = px / Wo;
-    int i = static_cast<int>(r % Ho);
-    int64_t n = r / Ho;
-    int64_t base = ((n * H + 2 * i) * W_ + 2 * j) * wpr + wi;
-    W w[4] = {in[base], in[base + wpr], in[base + (int64_t)W_ * wpr], in[base + (int64_t)W_ * wpr + wpr]};
-    W o = 0;
-    for (int l = 0; l < L; ++l) {
-      int best = lane_value(static_cast<uint32_t>(w[0] >> (l * lane_w)) & lm, bits, is_signed);
-      for (int k = 1; k < 4; ++k) {
-        int v = lane_value(static_cast<uint32_t>(w[k] >> (l * lane_w)) & lm, bits, is_signed);
-        best = v > best ? v : best;
-      }
-      o |= W(static_cast<uint32_t>(best) & lm) << (l * lane_w);
+__global__ void __launch_bounds__(kThreads) maxpool_field_kernel(const W *__restrict__ in, W *__restrict__ out, int Ho,
+                                                                 int Wo, int H, int W_, int wpr, int is_signed,
+                                                                 int rows, const FieldMasks<W> f) {
+  const int units = Wo * wpr;
+  const W flip = is_signed ? f.msb : W(0);
+  for (int row = blockIdx.x; row < rows; row += gridDim.x) {  // row = n * Ho + i
+    const int n = row / Ho, i = row - (row / Ho) * Ho;
+    const W *top = in + (static_cast<long long>(n) * H + 2 * i) * W_ * wpr;
+    const W *bot = top + static_cast<long long>(W_) * wpr;
+    W *dst = out + static_cast<long long>(row) * Wo * wpr;
+    for (int u = blockIdx.y * blockDim.x + threadIdx.x; u < units; u += gridDim.y * blockDim.x) {
+      const int j = u / wpr, q = u - (u / wpr) * wpr;
+      const int off = 2 * j * wpr + q;
+      const W m1 = field_max<W>(__ldcs(top + off), __ldcs(top + off + wpr), f, flip);
+      const W m2 = field_max<W>(__ldcs(bot + off), __ldcs(bot + off + wpr), f, flip);
+      dst[j * wpr + q] = field_max<W>(m1, m2, f, flip);
     }
-    out[t] = o;
   }
 }
 
 template <typename W>
 cudaError_t pool_dispatch(samd_fmt f, const void *in, void *out, int N, int C, int H, int W_, cudaStream_t s) {
   int wpr = static_cast<int>(words_per_row(f, C));
-  int64_t total = (int64_t)N * (H / 2) * (W_ / 2) * wpr;
-  int grid = grid_for(total, kThreads, sm_count() * 16);
   const W *pi = static_cast<const W *>(in);
   W *po = static_cast<W *>(out);
-  if (f.spacer != 0) {
-    maxpool_lane_kernel<W><<<grid, kThreads, 0, s>>>(pi, po, N, H, W_, wpr, f.bits, f.is_signed, f.bits + f.spacer,
-                                                     lanes_per_word(f));
-    return cudaGetLastError();
-  }
   const int Ho = H / 2, Wo = W_ / 2;
   constexpr int V16 = 16 / static_cast<int>(sizeof(W));
-  const bool vec = (wpr % V16) == 0;
+  const bool vec = f.spacer == 0 && (wpr % V16) == 0;
   const int units = Wo * (vec ? wpr / V16 : wpr);
   int gy = (units + kThreads - 1) / kThreads;
   if (gy > 65535) gy = 65535;
@@ -132,6 +120,11 @@ cudaError_t pool_dispatch(samd_fmt f, const void *in, void *out, int N, int C, i
   long long gx = (static_cast<long long>(sm_count()) * 8 + gy - 1) / gy;
   if (gx > rows) gx = rows;
   const dim3 pgrid(static_cast<unsigned>(gx), gy);
+  if (f.spacer != 0) {
+    maxpool_field_kernel<W><<<pgrid, kThreads, 0, s>>>(pi, po, Ho, Wo, H, W_, wpr, f.is_signed, rows,
+                                                       field_masks<W>(f));
+    return cudaGetLastError();
+  }
   switch (f.bits * 2 + (vec ? 1 : 0)) {
 #define SAMD_POOL_CASE(B)                                                                                   \
   case 2 * B:                                                                                               \

@@ -68,6 +68,52 @@ __device__ __forceinline__ int lane_value(uint32_t p, int bits, bool is_signed) 
 
 __device__ __forceinline__ int clamp_int(int v, int lo, int hi) { return v < lo ? lo : (v > hi ? hi : v); }
 
+// Masks over the lane fields of a format with permanent spacer bits (section
+// 2.1, Fig. 2): a field is `bits` data bits and `spacer` zero bits above
+// them, L fields per word.
+template <typename W>
+struct FieldMasks {
+  W lsb;    // bit 0 of every field
+  W msb;    // the top data bit (bits - 1) of every field
+  W carry;  // the first spacer bit (bit `bits`) of every field
+  W live;   // the data bits of every field
+  int bits, fw, L;  // data bits, field width, fields per word
+};
+
+template <typename W>
+inline FieldMasks<W> field_masks(samd_fmt f) {
+  FieldMasks<W> m;
+  m.bits = f.bits;
+  m.fw = f.bits + f.spacer;
+  m.L = lanes_per_word(f);
+  m.lsb = 0;
+  for (int i = 0; i < m.L; ++i) m.lsb |= W(1) << (i * m.fw);
+  m.msb = m.lsb << (f.bits - 1);
+  m.carry = m.lsb << f.bits;
+  m.live = m.lsb * ((W(1) << f.bits) - 1);
+  return m;
+}
+
+// Spread a mask of field bits at position p over the field's bits below p
+// (and p itself): m - (m >> p) sets bits [0, p), or-ing m keeps bit p.
+template <typename W>
+__device__ __forceinline__ W spread_down(W m, int p) {
+  return (m - (m >> p)) | m;
+}
+
+// Lane-wise max of two words of spacer-separated fields (spacer >= 1), flip
+// = the msb mask for signed lanes (offset binary orders like two's
+// complement), else 0: in (x | carry) - y every field computes 2^bits + x - y
+// > 0, so no borrow crosses a field and the carry bit stays set exactly
+// where x >= y.
+template <typename W>
+__device__ __forceinline__ W field_max(W a, W b, const FieldMasks<W> &f, W flip) {
+  const W x = a ^ flip, y = b ^ flip;
+  const W ge = ((x | f.carry) - y) & f.carry;
+  const W E = ge - (ge >> f.bits);  // the data bits of the lanes where x >= y
+  return (a & E) | (b & ~E & f.live);
+}
+
 }  // namespace samd
 
 // ---- launchers implemented in the kernel translation units ----------------

@@ -110,10 +110,11 @@ def test_requant_format_change(samd_lib, fa_t, fo_t):
     assert_status_clean()
 
 
-@pytest.mark.parametrize("spacer", (1, 2))
+@pytest.mark.parametrize("spacer", (1, 2, 4))
 @pytest.mark.parametrize("op", ("add", "sub", "mul", "relu"))
 def test_ops_with_spacer_bits(samd_lib, op, spacer):
-    for bits, signed, word_bits in [(3, True, 32), (4, False, 64), (7, True, 32), (1, False, 32)]:
+    for bits, signed, word_bits in [(3, True, 32), (4, False, 64), (7, True, 32), (1, False, 32), (2, True, 32),
+                                    (2, False, 64), (1, True, 32), (8, False, 64), (5, True, 64)]:
         f = samd.fmt(bits, signed, spacer, word_bits)
         n = 30011
         xv, xb = values_and_bytes(synth.seed_for("sx", op, bits, spacer), (n,), bits, signed)
@@ -123,6 +124,24 @@ def test_ops_with_spacer_bits(samd_lib, op, spacer):
             got = samd.elementwise(op, xw, yw if op != "relu" else None, f, n, saturate=sat and op != "relu")
             want_v = oracle.elementwise(op, xv, yv, bits=bits, signed=signed, saturate=sat and op != "relu")
             assert np.array_equal(np_words(got, word_bits), oracle.pack(want_v, bits, signed, spacer, word_bits))
+    assert_status_clean()
+
+
+@pytest.mark.parametrize("spacer", (1, 2, 5))
+@pytest.mark.parametrize("bits,signed,word_bits", [(1, False, 32), (3, True, 32), (4, False, 64), (7, True, 32),
+                                                   (8, True, 64), (2, True, 32)])
+def test_requant_same_format_with_spacer_bits(samd_lib, bits, signed, word_bits, spacer):
+    f = samd.fmt(bits, signed, spacer, word_bits)
+    n = 20011
+    xv, xb = values_and_bytes(synth.seed_for("rqs", bits, signed, spacer, word_bits), (n,), bits, signed)
+    xw = gpu_pack(xb, f, 1, n)
+    for shift in range(0, bits + 2):
+        got = samd.elementwise("requant", xw, None, f, n, shift=shift)
+        want_v = oracle.elementwise("requant", xv, bits=bits, signed=signed, bits_o=bits, signed_o=signed, shift=shift)
+        assert np.array_equal(np_words(got, word_bits), oracle.pack(want_v, bits, signed, spacer, word_bits)), shift
+    got = samd.elementwise("relu", xw, None, f, n)
+    want = oracle.pack(oracle.elementwise("relu", xv, bits=bits, signed=signed), bits, signed, spacer, word_bits)
+    assert np.array_equal(np_words(got, word_bits), want)
     assert_status_clean()
 
 
