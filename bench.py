@@ -274,61 +274,109 @@ def build_layers(layers, dev):
 
 
 def time_packed_ops(dev, flush):
-    """GB/s of pack/unpack, the five elementwise ops and max-pool at 2^28 lanes."""
+    """GB/s of pack/unpack, the five elementwise ops (spacer-free, and with one
+    permanent spacer bit per lane) and max-pool at 2^28 lanes.
+
+    Each figure times 8 launches back to back, rotating over independent sets
+    of input and output buffers whose total is at least twice the L2: each
+    launch finds its inputs in DRAM, and the write-back of one launch's output
+    happens during the next one, inside the timed region (only the last
+    launch's may escape it). L2 is flushed before the first launch."""
     import torch
 
     from paper_1809_10572_gb300 import samd, synth, workloads
 
     n = workloads.ELEMENTWISE_N
     res = {}
+    reps = 8
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
 
-    def timed(fn, nbytes, reps=3):
+    def n_sets(set_bytes):
+        return max(2, -(-2 * L2_BYTES // set_bytes) + 1)
+
+    def timed(fns, nbytes):
         ts = []
-        for _ in range(reps):
+        for _ in range(3):
             flush()
             start.record()
-            fn()
+            for i in range(reps):
+                fns[i % len(fns)]()
             end.record()
             end.synchronize()
             ts.append(start.elapsed_time(end) * 1e-3)
-        return nbytes / statistics.median(ts) / 1e9
+        return reps * nbytes / statistics.median(ts) / 1e9
 
-    launches = 0
-    for signed in (False, True):
-        tag = "s" if signed else "u"
-        for b in range(1, 9):
-            f = samd.fmt(b, signed)
-            xb = synth.to_bytes_t(synth.lanes_t(synth.seed_for("ewx", b, signed), (n,), b, signed, device=dev))
-            xw = samd.pack(xb, f)
-            yw = samd.pack(synth.to_bytes_t(synth.lanes_t(synth.seed_for("ewy", b, signed), (n,), b, signed,
-                                                          device=dev)), f)
-            out = torch.empty_like(xw)
-            wbytes = xw.numel() * 4
-            res.setdefault("pack", {}).setdefault(tag, []).append(
-                timed(lambda: samd.samd_pack(f, xb, out, 1, n), n + wbytes))
-            res.setdefault("unpack", {}).setdefault(tag, []).append(
-                timed(lambda: samd.samd_unpack(f, xw, xb, 1, n), n + wbytes))
-            for op in workloads.ELEMENTWISE_OPS:
-                binary = op in ("add", "sub", "mul")
-                nb = (3 if binary else 2) * wbytes
-                res.setdefault(op, {}).setdefault(tag, []).append(
-                    timed(lambda: samd.samd_elementwise(op, f, xw, yw if binary else None, f, out, n,
-                                                        1 if op == "requant" else 0, 0), nb))
-            launches += 3 * 7
-            del xb, xw, yw, out
+    for spacer in (0, 1):
+        for signed in (False, True):
+            tag = ("s" if signed else "u") + ("_spacer1" if spacer else "")
+            for b in range(1, 9 - spacer):
+                f = samd.fmt(b, signed, spacer)
+                xb = synth.to_bytes_t(synth.lanes_t(synth.seed_for("ewx", b, signed), (n,), b, signed, device=dev))
+                xw = samd.pack(xb, f)
+                wbytes = xw.numel() * 4
+                ns = n_sets(2 * wbytes + (n if spacer == 0 else 0))
+                xws = [xw] + [xw.clone() for _ in range(ns - 1)]
+                yws = [samd.pack(synth.to_bytes_t(synth.lanes_t(synth.seed_for("ewy", b, signed, k), (n,), b, signed,
+                                                                device=dev)), f) for k in range(ns)]
+                outs = [torch.empty_like(xw) for _ in range(ns)]
+                if spacer == 0:
+                    xbs = [xb] + [xb.clone() for _ in range(ns - 1)]
+                    res.setdefault("pack", {}).setdefault(tag, []).append(timed(
+                        [lambda k=k: samd.samd_pack(f, xbs[k], outs[k], 1, n) for k in range(ns)], n + wbytes))
+                    res.setdefault("unpack", {}).setdefault(tag, []).append(timed(
+                        [lambda k=k: samd.samd_unpack(f, xws[k], xbs[k], 1, n) for k in range(ns)], n + wbytes))
+                    del xbs
+                for op in workloads.ELEMENTWISE_OPS:
+                    binary = op in ("add", "sub", "mul")
+                    nb = (3 if binary else 2) * wbytes
+                    res.setdefault(op, {}).setdefault(tag, []).append(timed(
+                        [lambda k=k: samd.samd_elementwise(op, f, xws[k], yws[k] if binary else None, f, outs[k], n,
+                                                           1 if op == "requant" else 0, 0) for k in range(ns)], nb))
+                del xb, xw, xws, yws, outs
     # 2x2 max-pool on VGG-16 block-1 activations (224 x 224 x 64, u4): at
-    # batch 128 (258 MB moved, HBM-bound) and at the workload's batch 16
-    # (32 MB, short enough that launch and ramp-up show)
+    # batch 128 (258 MB moved) and at the workload's batch 16 (32 MB)
     f = samd.fmt(4, False)
     C, H, W = 64, 224, 224
     for N, key in ((128, "maxpool2x2"), (16, "maxpool2x2_batch16")):
         xw = samd.pack(synth.to_bytes_t(synth.lanes_t(5, (N * H * W, C), 4, False, device=dev)), f)
         out = samd.empty_words(f, N * H * W // 4, C, dev)
         nb = (xw.numel() + out.numel()) * 4
-        res[key] = {"u": [timed(lambda: samd.samd_maxpool2x2(f, xw, out, N, C, H, W), nb)]}
-        del xw, out
+        ns = n_sets(nb)
+        xs = [xw] + [xw.clone() for _ in range(ns - 1)]
+        outs = [out] + [torch.empty_like(out) for _ in range(ns - 1)]
+        res[key] = {"u": [timed([lambda k=k: samd.samd_maxpool2x2(f, xs[k], outs[k], N, C, H, W) for k in range(ns)],
+                                nb)]}
+        del xw, out, xs, outs
     return res
+
+
+def time_nchw_widemul(dev):
+    """The paper's wide-multiply engine (NCHW packed along W, CUDA cores) on
+    the sweep's 3x3 C64 -> 64 56x56 layer at batch 8, for the lane widths whose
+    kernel row fits one 64-bit word: effective MAC/s, beside the tensor-core
+    path's per-layer rates."""
+    import torch
+
+    from paper_1809_10572_gb300 import samd, synth
+
+    shape = samd.ConvShape(8, 64, 56, 56, 64)
+    out = {}
+    for b, sa, sw in [(1, False, False), (1, True, True), (2, False, False), (2, True, True), (3, True, True),
+                      (4, False, True), (4, True, True), (5, True, True)]:
+        fa, fw = samd.fmt(b, sa), samd.fmt(b, sw)
+        desc = shape.desc(samd.SAMD_NCHW)
+        if samd.samd_conv2d_operand_bits(desc, fa, fw) == 0:
+            continue
+        a = samd.pack(synth.to_bytes_t(synth.lanes_t(1, (shape.N * shape.C * shape.H, shape.W), b, sa, device=dev)),
+                      fa)
+        w = samd.pack(synth.to_bytes_t(synth.lanes_t(2, (shape.K * shape.C * shape.R, shape.S), b, sw, device=dev)),
+                      fw)
+        ws = torch.empty(samd.samd_conv2d_workspace_size(desc, fa, fw), dtype=torch.uint8, device=dev)
+        packed = samd.empty_words(fa, shape.N * shape.K * shape.Ho, shape.Wo, dev)
+        run = lambda: samd.samd_conv2d(desc, fa, a, fw, w, None, fa, packed, b, ws)
+        t = _best_time(run, reps=5)
+        out[f"b{b}_{'s' if sa else 'u'}{'s' if sw else 'u'}"] = shape.macs / t
+    return out
 
 
 def csrc_digest():
@@ -559,7 +607,11 @@ def run_samd(args, layers):
                                        "peak_source": "measured" if peaks.get("hbm_gbs") else "fallback",
                                        "min_frac": min(fr), "median_frac": statistics.median(fr), "max_frac": max(fr),
                                        "n": 2 ** 28, "word_bits": 32,
-                                       "bytes": "each input word read once + each output word written once"}
+                                       "bytes": "each input word read once + each output word written once",
+                                       "timing": "8 launches back to back over rotating buffer sets of more than "
+                                                 "twice the L2 (write-back of each output inside the timed region); "
+                                                 "L2 flushed first"}
+        line["nchw_widemul_mac_s"] = time_nchw_widemul(dev)
     line["clocks"] = clk
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         v, cores, sample = cpu_oracle_rate(layers, args.cpu_seconds)

@@ -665,18 +665,27 @@ samd_status conv2d_nhwc(const samd_conv_desc *d, samd_fmt fa, const void *act, s
   return conv2d_run(d, fa, fw, act, workspace, workspace_bytes, acc_out, fplan, packed_out, shift, s);
 }
 
-samd_status conv2d_nhwc_noalloc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
-                                int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, cudaStream_t s) {
-  conv::Plan p;
-  samd_status st = conv::make_plan(d, fa, fw, packed_out ? fo : conv::none_fmt(), p);
-  if (st != SAMD_OK) return st;
-  // the widened weights of this call (shape, formats, output format) must fit
-  if (p.ws_bytes > kNoallocScratchBytes) return SAMD_EUNSUP;
+samd_status conv2d_noalloc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
+                           int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, cudaStream_t s) {
+  size_t need = 0;
+  if (d->layout == SAMD_NCHW) {
+    samd_status st = conv2d_nchw_check(d, fa, fw, packed_out ? fo : conv::none_fmt(), &need);
+    if (st != SAMD_OK) return st;
+  } else {
+    conv::Plan p;
+    samd_status st = conv::make_plan(d, fa, fw, packed_out ? fo : conv::none_fmt(), p);
+    if (st != SAMD_OK) return st;
+    need = p.ws_bytes;
+  }
+  // the scratch this call needs (for its shape, formats and output format) must fit
+  if (need > kNoallocScratchBytes) return SAMD_EUNSUP;
   void *scratch = nullptr;
   if (conv::g_scratch_addr.get(reinterpret_cast<const void *>(&g_noalloc_scratch), &scratch) != cudaSuccess)
     return SAMD_ECUDA;
-  // prepare writes every byte of the widened weights that run then reads, so
-  // nothing left over from an earlier call is ever used
+  // the calls below write every byte of scratch they then read, so nothing
+  // left over from an earlier call is ever used
+  if (d->layout == SAMD_NCHW)
+    return conv2d_nchw(d, fa, act, fw, wt, acc_out, fo, packed_out, shift, scratch, kNoallocScratchBytes, s);
   return conv2d_nhwc(d, fa, act, fw, wt, acc_out, fo, packed_out, shift, scratch, kNoallocScratchBytes, s);
 }
 

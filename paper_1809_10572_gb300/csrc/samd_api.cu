@@ -84,6 +84,12 @@ size_t samd_conv2d_workspace_size(const samd_conv_desc *d, samd_fmt fa, samd_fmt
   if (d->N < 0 || d->C < 1 || d->H < 1 || d->W < 1 || d->K < 1 || d->R < 1 || d->S < 1 || d->stride < 1 ||
       d->pad < 0)
     return 0;
+  if (d->layout == SAMD_NCHW) {
+    size_t ws = 0;
+    if (fa.spacer != 0 || fw.spacer != 0 || d->R > 16 || d->S > 16) return 0;
+    return conv2d_nchw_check(d, fa, fw, samd_fmt{0, 0, 0, 0}, &ws) == SAMD_OK ? ws : 0;
+  }
+  if (d->layout != SAMD_NHWC) return 0;
   return conv2d_workspace_size(d, fa, fw);
 }
 
@@ -98,6 +104,8 @@ int samd_conv2d_operand_bits(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw) 
   if (d->N < 0 || d->C < 1 || d->H < 1 || d->W < 1 || d->K < 1 || d->R < 1 || d->S < 1 || d->stride < 1 ||
       d->pad < 0 || d->R > 16 || d->S > 16)
     return 0;
+  if (d->layout == SAMD_NCHW) return conv2d_nchw_check(d, fa, fw, samd_fmt{0, 0, 0, 0}, nullptr) == SAMD_OK ? 64 : 0;
+  if (d->layout != SAMD_NHWC) return 0;
   return conv2d_operand_bits(d, fa, fw);
 }
 
@@ -114,9 +122,9 @@ samd_status conv_common_checks(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw
       d->pad < 0)
     return SAMD_ESHAPE;
   if (d->H + 2 * d->pad < d->R || d->W + 2 * d->pad < d->S) return SAMD_ESHAPE;
-  if (d->layout != SAMD_NHWC) return SAMD_EUNSUP;
   if (fa.spacer != 0 || fw.spacer != 0) return SAMD_EUNSUP;
   if (d->R > 16 || d->S > 16) return SAMD_EUNSUP;
+  if (d->layout == SAMD_NCHW) return conv2d_nchw_check(d, fa, fw, fo, nullptr);  // wide-multiply engine limits
   return conv2d_check(d, fa, fw);  // exactness bound of the accumulation
 }
 }  // namespace
@@ -133,6 +141,9 @@ samd_status samd_conv2d(const samd_conv_desc *d, samd_fmt fa, const void *act, s
   if (!aligned16(act) || !aligned16(wt) || !aligned16(workspace) || (acc_out && !aligned16(acc_out)) ||
       (packed_out && !aligned16(packed_out)))
     return SAMD_EALIGN;
+  if (d->layout == SAMD_NCHW)
+    return conv2d_nchw(d, fa, act, fw, wt, acc_out, fo, packed_out, shift, workspace, workspace_bytes,
+                       reinterpret_cast<cudaStream_t>(stream));
   return conv2d_nhwc(d, fa, act, fw, wt, acc_out, fo, packed_out, shift, workspace, workspace_bytes,
                      reinterpret_cast<cudaStream_t>(stream));
 }
@@ -148,7 +159,7 @@ samd_status samd_conv2d_noalloc(const samd_conv_desc *d, samd_fmt fa, const void
   if (!aligned16(act) || !aligned16(wt) || (acc_out && !aligned16(acc_out)) ||
       (packed_out && !aligned16(packed_out)))
     return SAMD_EALIGN;
-  return conv2d_nhwc_noalloc(d, fa, act, fw, wt, acc_out, fo, packed_out, shift,
+  return conv2d_noalloc(d, fa, act, fw, wt, acc_out, fo, packed_out, shift,
                              reinterpret_cast<cudaStream_t>(stream));
 }
 
@@ -156,6 +167,7 @@ samd_status samd_conv2d_prepare(const samd_conv_desc *d, samd_fmt fa, samd_fmt f
                                 void *prepared, size_t prepared_bytes, samd_stream_t stream) {
   samd_status st = conv_common_checks(d, fa, fw, fo, 0);
   if (st != SAMD_OK) return st;
+  if (d->layout != SAMD_NHWC) return SAMD_EUNSUP;  // the NCHW engine widens its operands on every call
   if (!wt || !prepared) return SAMD_EINVAL;
   if (!aligned16(wt) || !aligned16(prepared)) return SAMD_EALIGN;
   return conv2d_prepare(d, fa, fw, wt, fo, prepared, prepared_bytes, reinterpret_cast<cudaStream_t>(stream));
@@ -168,6 +180,7 @@ samd_status samd_conv2d_prepared(const samd_conv_desc *d, samd_fmt fa, const voi
   if (packed_out && fo.bits == 0) return SAMD_EINVAL;
   samd_status st = conv_common_checks(d, fa, fw, fo, packed_out ? shift : 0);
   if (st != SAMD_OK) return st;
+  if (d->layout != SAMD_NHWC) return SAMD_EUNSUP;
   if (d->N == 0) return SAMD_OK;
   if (!act || !prepared) return SAMD_EINVAL;
   if (!aligned16(act) || !aligned16(prepared) || (acc_out && !aligned16(acc_out)) ||

@@ -139,8 +139,13 @@ size_t conv2d_workspace_size(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw);
 int conv2d_operand_bits(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw);
 void conv2d_set_min_tiles_per_cta(int tiles);
 constexpr size_t kNoallocScratchBytes = size_t(8) << 20;  // static scratch of samd_conv2d_noalloc
-samd_status conv2d_nhwc_noalloc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
+samd_status conv2d_noalloc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
                                 int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, cudaStream_t s);
+// NCHW packed along W: the wide-multiply engine of widemul.cu
+samd_status conv2d_nchw_check(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fmt fo, size_t *ws_bytes);
+samd_status conv2d_nchw(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
+                        int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, void *workspace,
+                        size_t workspace_bytes, cudaStream_t s);
 cudaError_t read_device_status(int *status, int reset, cudaStream_t s);
 cudaError_t selftest_wait_timeout(uint64_t limit_ns, cudaStream_t s);
 }  // namespace samd

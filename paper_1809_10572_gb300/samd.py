@@ -321,6 +321,23 @@ def conv2d(act, wt, shape: ConvShape, fa: samd_fmt, fw: samd_fmt, fo: samd_fmt |
     return acc, packed
 
 
+def conv2d_nchw(act, wt, shape: ConvShape, fa: samd_fmt, fw: samd_fmt, fo: samd_fmt | None = None, shift: int = 0,
+                want_acc: bool = True, workspace=None, stream=None):
+    """NCHW packed along W (rows of W lanes; weights [K][C][R] rows of S lanes);
+    returns (int32 acc [N,K,Ho,Wo] or None, packed output rows of Wo lanes or None)."""
+    dev = act.device
+    desc = shape.desc(SAMD_NCHW)
+    acc = torch.empty((shape.N, shape.K, shape.Ho, shape.Wo), dtype=torch.int32, device=dev) if want_acc else None
+    packed = empty_words(fo, shape.N * shape.K * shape.Ho, shape.Wo, dev) if fo is not None else None
+    if workspace is None:
+        nbytes = samd_conv2d_workspace_size(desc, fa, fw)
+        if nbytes == 0:
+            raise SamdError(SAMD_EUNSUP, "samd_conv2d_workspace_size")
+        workspace = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    samd_conv2d(desc, fa, act, fw, wt, acc, fo, packed, shift, workspace, stream=stream)
+    return acc, packed
+
+
 class PreparedConv:
     """A convolution layer whose weights were widened once (samd_conv2d_prepare)."""
 

@@ -76,8 +76,12 @@ def test_conv_argument_checks(lib):
     d = samd.ConvShape(1, 16, 8, 8, 16).desc()
     assert lib.samd_conv2d(None, fa, 16, fw, 16, 16, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_EINVAL
     assert lib.samd_conv2d(ctypes.byref(d), fa, 16, fw, 16, None, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_EINVAL
+    # NCHW (the wide-multiply engine): stride 1 only; pointers checked before any launch
     nchw = samd.ConvShape(1, 16, 8, 8, 16).desc(samd.SAMD_NCHW)
-    assert lib.samd_conv2d(ctypes.byref(nchw), fa, 16, fw, 16, 16, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_EUNSUP
+    assert lib.samd_conv2d(ctypes.byref(nchw), fa, 16, fw, 24, 16, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_EALIGN
+    nchw2 = samd.ConvShape(1, 16, 8, 8, 16, stride=2).desc(samd.SAMD_NCHW)
+    assert lib.samd_conv2d(ctypes.byref(nchw2), fa, 16, fw, 16, 16, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_EUNSUP
+    assert lib.samd_conv2d_prepare(ctypes.byref(nchw), fa, fw, 16, fa, 16, 1 << 20, None) == samd.SAMD_EUNSUP
     bad = samd.ConvShape(1, 16, 2, 2, 16, R=5, S=5, pad=1).desc()
     assert lib.samd_conv2d(ctypes.byref(bad), fa, 16, fw, 16, 16, fa, None, 0, 16, 1 << 20, None) == samd.SAMD_ESHAPE
     # u8 x s8 over 3x3x512 taps: even split weight digits exceed 2^24 (4608 * 255 * 16)
@@ -118,6 +122,25 @@ def test_conv_operand_type_query(lib):
     assert samd.samd_conv2d_operand_bits(d, samd.fmt(4, False, spacer=1), samd.fmt(4, True)) == 0
     assert samd.samd_conv2d_operand_bits(samd.ConvShape(1, 0, 8, 8, 16).desc(), samd.fmt(4, False),
                                          samd.fmt(4, True)) == 0
+
+
+def test_nchw_wide_multiply_plan():
+    """Section 5.1 engine: fields of F = bits(R*S*C*max|a|*max|w|) + 1 bits,
+    nx = floor(64 / F) inputs per word, the kernel row in one word (S*F <= 64).
+    u4 x s4 over 3x3x16: bound 17280 (15 bits) -> F = 16, nx = 4; an 8-wide
+    output row needs the 10 coefficients of the full 1D convolution, G = 3
+    words per input row. Workspace: 8 bytes x (N*C*H*G + K*C*R)."""
+    fa, fw = samd.fmt(4, False), samd.fmt(4, True)
+    d = samd.ConvShape(1, 16, 8, 8, 16).desc(samd.SAMD_NCHW)
+    assert samd.samd_conv2d_workspace_size(d, fa, fw) == 8 * (1 * 16 * 8 * 3 + 16 * 16 * 3)
+    assert samd.samd_conv2d_operand_bits(d, fa, fw) == 64
+    # u8 x s8 over 3x3x64: bound 576 * 255 * 128 = 18.8 M (25 bits) -> F = 26, 3 x 26 > 64
+    big = samd.ConvShape(1, 64, 8, 8, 16).desc(samd.SAMD_NCHW)
+    assert samd.samd_conv2d_operand_bits(big, samd.fmt(8, False), samd.fmt(8, True)) == 0
+    assert samd.samd_conv2d_workspace_size(big, samd.fmt(8, False), samd.fmt(8, True)) == 0
+    # the same sums over 1x2 kernels fit (2 x 26 <= 64)
+    ok = samd.ConvShape(1, 64, 8, 8, 16, R=1, S=2, pad=0).desc(samd.SAMD_NCHW)
+    assert samd.samd_conv2d_operand_bits(ok, samd.fmt(8, False), samd.fmt(8, True)) == 64
 
 
 def test_min_tiles_per_cta_setting(lib):
