@@ -25,6 +25,12 @@ SAMD_STUB(launch_conv_f8_w64_b4) SAMD_STUB(launch_conv_f8_w64_b5)
 
 namespace samd {
 int sm_count() { return 152; }  // defined in samd_api.cu, not linked here
+// the NCHW path lives in widemul.cu, not linked here
+samd_status conv2d_nchw_check(const samd_conv_desc *, samd_fmt, samd_fmt, samd_fmt, size_t *) { return SAMD_EUNSUP; }
+samd_status conv2d_nchw(const samd_conv_desc *, samd_fmt, const void *, samd_fmt, const void *, int32_t *, samd_fmt,
+                        void *, int, void *, size_t, cudaStream_t) {
+  return SAMD_EUNSUP;
+}
 }  // namespace samd
 
 #include <cstdio>
