@@ -198,6 +198,8 @@ struct Plan {
   int nseg, seg_rows, seg_used, row_step;  // halo geometry (see ConvArgs)
   long long grid_m;                        // 128-position tiles along the output
   int stages_a, b_resident;
+  int gdepth;  // HALO: packed staging slots (items gathered gdepth - 1 ahead of the widening)
+  int e_stage; // kEpiStageBytes at off_e stage the epilogue's 3/5/6-bit packed rows
   long long M;
   long long bound;  // R*S*C * max|a| * max|w|: no accumulator exceeds it
   uint32_t tmem_cols;
@@ -299,6 +301,7 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
     const int bmt = BM * hv;
     p.hv = hv;
     p.halo = 0;
+    p.gdepth = 2;
     p.b_resident = 0;
     p.stages_a = 0;
     p.nseg = p.seg_rows = p.seg_used = p.row_step = 0;
@@ -328,11 +331,23 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
       const double waste = static_cast<double>(d->N) * p.Hv * p.Wp / static_cast<double>(p.M);
       const size_t halo_bytes = round_up(static_cast<size_t>(halo_rows) * p.row_bytes, 1024);
       const size_t stage_g = round_up(static_cast<size_t>(halo_rows) * srow, 16);
-      const size_t fixed = 2 * halo_bytes + 2 * stage_g + e_bytes + 1024;
       const int ntiles_b = p.nck * p.taps;
-      if (halo_rows > kMaxHaloRows || waste > 1.16 || fixed + 2 * bst + bar_bytes(2, 2) > kBudget) return false;
-      const bool res = p.nblocks == 1 && fixed + ntiles_b * bst + bar_bytes(ntiles_b, 2) <= kBudget;
-      if (need_resident && !res) return false;
+      if (halo_rows > kMaxHaloRows || waste > 1.16) return false;
+      // The deepest packed staging ring (4, 3 or 2 items) that fits: with
+      // depth D the gathers run D - 1 items ahead of the widening, which
+      // hides the global-memory latency behind D - 1 items of MMA work.
+      size_t fixed = 0;
+      bool res = false;
+      int depth = 4;
+      for (; depth >= 2; --depth) {
+        fixed = 2 * halo_bytes + depth * stage_g + e_bytes + 1024;
+        if (fixed + 2 * bst + bar_bytes(2, 2) > kBudget) continue;
+        res = p.nblocks == 1 && fixed + ntiles_b * bst + bar_bytes(ntiles_b, 2) <= kBudget;
+        if (need_resident && !res) continue;
+        break;
+      }
+      if (depth < 2) return false;
+      p.gdepth = depth;
       p.halo = 1;
       p.nchunks = ntiles_b;
       p.Kpad = ntiles_b * BK;
@@ -346,7 +361,7 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
       }
       p.op_stride = static_cast<uint32_t>(halo_bytes);
       p.g_stride = static_cast<uint32_t>(stage_g);
-      finish(2 * halo_bytes, 2 * stage_g, 2);
+      finish(2 * halo_bytes, depth * stage_g, 2);
       return true;
     }
     const size_t tile_bytes = static_cast<size_t>(bmt) * p.row_bytes;
@@ -383,6 +398,16 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
       placed = place(halo, hv, need_res != 0);
     }
   if (!placed) return SAMD_EUNSUP;  // operand tiles do not fit (not reached for N <= 256)
+  // 3-, 5- and 6-bit packed outputs (32-bit words, no spacer) stage their
+  // rows in shared memory when that fits beside the placement chosen above
+  // (which it never changes), so that stores are contiguous within a row.
+  p.e_stage = 0;
+  if ((fo.bits == 3 || fo.bits == 5 || fo.bits == 6) && fo.spacer == 0 && fo.word_bits == 32 &&
+      p.smem_bytes + round_up(kEpiStageBytes, 16) <= kBudget) {
+    p.e_stage = 1;
+    p.off_bar = static_cast<uint32_t>(round_up(p.off_e + kEpiStageBytes, 16));
+    p.smem_bytes = 1024 + p.off_bar + bar_bytes(p.stages, p.halo ? 2 : p.stages_a);
+  }
   uint32_t cols = 32;
   while (cols < static_cast<uint32_t>(2 * p.hv * p.mma_n)) cols <<= 1;  // two accumulators of hv halves
   p.tmem_cols = cols;
@@ -399,10 +424,11 @@ bool layout_ok(const Plan &p) {
   const size_t op_bytes = NO * p.op_stride;
   const size_t bars = (2 * static_cast<size_t>(p.stages) + 2 * NO + 5) * 8 + 4;
   return p.stages >= 1 && NO >= 2 && op_bytes <= p.off_b &&
-         p.off_b + static_cast<size_t>(p.stages) * p.b_bytes <= p.off_g && p.off_g + 2 * p.g_stride <= p.off_e &&
+         p.off_b + static_cast<size_t>(p.stages) * p.b_bytes <= p.off_g && p.off_g + static_cast<size_t>(p.halo ? p.gdepth : 2) * p.g_stride <= p.off_e &&
          p.off_e <= p.off_bar && 1023 + p.off_bar + bars <= p.smem_bytes && p.op_stride % 1024 == 0 &&
          p.off_b % 1024 == 0 && p.b_bytes % 1024 == 0 && p.off_bar % 8 == 0 && 2 * p.hv * p.mma_n <= 512 &&
-         (p.hv == 1 || p.hv == 2);
+         (p.hv == 1 || p.hv == 2) && (!p.halo || (p.gdepth >= 2 && p.gdepth <= 4)) &&
+         (!p.e_stage || p.off_e + kEpiStageBytes <= p.off_bar);
 }
 
 // Device address of a __device__ symbol in the current context, looked up
@@ -622,7 +648,9 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   a.b_bytes = p.b_bytes;
   a.off_g = p.off_g;
   a.g_stride = p.g_stride;
+  a.gdepth = p.gdepth;
   a.off_e = p.off_e;
+  a.e_stage = p.e_stage;
   a.off_bar = p.off_bar;
   // A small layer gives each CTA at least T reference tiles of work (T from
   // samd_conv2d_set_min_tiles_per_cta; a reference tile is 128 positions of

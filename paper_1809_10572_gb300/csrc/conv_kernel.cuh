@@ -48,6 +48,11 @@ constexpr int kEpiWarps = 8;                       // epilogue
 constexpr int kProdThreads = 32 * kProdWarps;
 constexpr int kThreads = 32 * (2 + kProdWarps + kEpiWarps);
 constexpr int kFirstEpiWarp = 2 + kProdWarps;
+// Optional epilogue staging (ConvArgs::e_stage): per epilogue warp 32 rows of
+// one packing period (at most 32 words), rows kEpiPitch words apart (odd, so
+// that 32 lanes writing one word of their own rows hit 32 banks).
+constexpr int kEpiPitch = 33;
+constexpr uint32_t kEpiStageBytes = kEpiWarps * 32 * kEpiPitch * 4;
 
 template <bool FP8>
 struct OpTraits {
@@ -156,6 +161,7 @@ struct ConvArgs {
   int gather_vec;   // AGather::vec
   int gather_win;   // AGather::issue_win (1x1 layers whose chunks are not aligned vectors)
   int g_row;        // GATHER staging row pitch in bytes
+  int gdepth;       // HALO: packed staging slots; gathers run gdepth - 1 items ahead
   long long act_bytes;  // bytes of the activation tensor (the windows stop at its end)
   uint32_t tmem_cols;
   int out_bits, out_signed, out_lane_w, out_L, out_word64, out_wpr;
@@ -182,6 +188,7 @@ struct ConvArgs {
   // shared memory carve-up (bytes from the 1024-byte-aligned base)
   uint32_t op_stride;  // one halo buffer or one A tile
   uint32_t off_b, b_bytes, off_g, g_stride, off_e, off_bar;
+  int e_stage;  // 1: kEpiStageBytes at off_e stage the 3/5/6-bit packed rows (epilogue_row_period_staged)
 };
 
 __device__ __forceinline__ uint32_t hsub2_bits(uint32_t a, uint32_t b) {
@@ -752,6 +759,74 @@ __device__ __forceinline__ void epilogue_row_period(const ConvArgs &args, uint32
   }
 }
 
+// epilogue_row_period with the stores staged: a warp's 32 rows of one
+// period (PW = lcm(32, L) / L words per row, 16 or 32) go to the warp's
+// shared-memory area first, and the warp then writes them out row by row,
+// PW consecutive words of 32 / PW rows per store instruction, instead of
+// every thread storing its own row one word at a time (32 rows, 32 sectors,
+// per instruction). Every word of a period is computed (channels past the
+// block's last read as the biased zero; 32-column groups wholly past it are
+// skipped), and only the block's words are stored.
+template <int OB, bool OS>
+__device__ __forceinline__ void epilogue_row_period_staged(const ConvArgs &args, uint32_t taddr, bool row_valid,
+                                                           long long m, int nb, uint32_t *stg) {
+  constexpr int L = 32 / OB;
+  constexpr int G = L / gcd_c(32, L);  // lcm(32, L) / 32
+  constexpr int PW = 32 * G / L;       // words per row and period
+  constexpr int RPI = 32 / PW;         // rows per store instruction
+  static_assert(PW * RPI == 32, "a period is 16 or 32 words");
+  constexpr int32_t lo = OS ? -(1 << (OB - 1)) : 0, hi = OS ? (1 << (OB - 1)) - 1 : (1 << OB) - 1;
+  constexpr int32_t blo = kMagicBits + lo, bhi = kMagicBits + hi;
+  constexpr uint32_t omask = (1u << OB) - 1;
+  const int lane = threadIdx.x & 31;
+  const int ch0 = nb * args.NBc;
+  const int nvalid = args.K - ch0 < args.NBc ? args.K - ch0 : args.NBc;
+  const int nwords = (nvalid + L - 1) / L;  // the block's words in a row
+  const float scale = args.out_scale;
+  const unsigned vmask = __ballot_sync(0xffffffffu, row_valid);
+  uint32_t *const out = static_cast<uint32_t *>(args.packed_out) + ch0 / L;
+  uint32_t *const mine = stg + lane * kEpiPitch;
+  for (int c0 = 0, wbase = 0; c0 < nvalid; c0 += 32 * G, wbase += PW) {
+    uint32_t cur = 0;
+    bool open = false;
+    int wcur = 0;  // words of this period staged so far
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const int col = c0 + 32 * g;
+      if (col >= nvalid) break;
+      uint32_t r[32];
+      ptx::tmem_ld_32x32b_x32(taddr + col, r);
+      ptx::tmem_wait_ld();
+#pragma unroll
+      for (int k = 0; k < 32; ++k) {
+        const int q = 32 * g + k;  // channel within the period (compile-time after unrolling)
+        const int l = q % L;
+        int32_t t = floor_scaled_biased(__uint_as_float(r[k]), scale);
+        t = t < blo ? blo : (t > bhi ? bhi : t);
+        if (col + k >= nvalid) t = kMagicBits;
+        cur |= (static_cast<uint32_t>(t) & omask) << (l * OB);
+        open = true;
+        if (l == L - 1) {
+          mine[wcur++] = cur;
+          cur = 0;
+          open = false;
+        }
+      }
+    }
+    if (open) mine[wcur] = cur;  // the row's last, partial word
+    __syncwarp();
+    const int nw = nwords - wbase < PW ? nwords - wbase : PW;  // this period's words inside the block
+    const int wi = lane % PW;
+#pragma unroll 4
+    for (int r0 = 0; r0 < 32; r0 += RPI) {
+      const int rr = r0 + lane / PW;
+      const long long mr = __shfl_sync(0xffffffffu, m, rr);
+      if (((vmask >> rr) & 1u) && wi < nw) out[mr * args.out_wpr + wbase + wi] = stg[rr * kEpiPitch + wi];
+    }
+    __syncwarp();
+  }
+}
+
 // Every other case, 16 columns at a time: split digits (acc = 16 hi + lo),
 // int32 outputs, accumulators too large for the fma path.
 template <typename WO>
@@ -810,7 +885,7 @@ __device__ __forceinline__ void epilogue_row_general(const ConvArgs &args, uint3
 }
 
 __device__ __forceinline__ void epilogue_row(const ConvArgs &args, uint32_t taddr, bool row_valid, long long m,
-                                             int nb) {
+                                             int nb, uint32_t *estage) {
   const bool fast = args.packed_out && !args.acc_out && !args.split && args.fast_req;
   if (fast && args.out_lane_w == args.out_bits && (!args.out_word64 || (args.out_bits & (args.out_bits - 1)) == 0)) {
     switch (args.out_bits * 2 + (args.out_signed ? 1 : 0)) {
@@ -818,14 +893,44 @@ __device__ __forceinline__ void epilogue_row(const ConvArgs &args, uint32_t tadd
       case 3: epilogue_row_spec<1, true>(args, taddr, row_valid, m, nb); return;
       case 4: epilogue_row_spec<2, false>(args, taddr, row_valid, m, nb); return;
       case 5: epilogue_row_spec<2, true>(args, taddr, row_valid, m, nb); return;
-      case 6: epilogue_row_period<3, false>(args, taddr, row_valid, m, nb); return;
-      case 7: epilogue_row_period<3, true>(args, taddr, row_valid, m, nb); return;
+      case 6:
+        if (estage)
+          epilogue_row_period_staged<3, false>(args, taddr, row_valid, m, nb, estage);
+        else
+          epilogue_row_period<3, false>(args, taddr, row_valid, m, nb);
+        return;
+      case 7:
+        if (estage)
+          epilogue_row_period_staged<3, true>(args, taddr, row_valid, m, nb, estage);
+        else
+          epilogue_row_period<3, true>(args, taddr, row_valid, m, nb);
+        return;
       case 8: epilogue_row_spec<4, false>(args, taddr, row_valid, m, nb); return;
       case 9: epilogue_row_spec<4, true>(args, taddr, row_valid, m, nb); return;
-      case 10: epilogue_row_period<5, false>(args, taddr, row_valid, m, nb); return;
-      case 11: epilogue_row_period<5, true>(args, taddr, row_valid, m, nb); return;
-      case 12: epilogue_row_period<6, false>(args, taddr, row_valid, m, nb); return;
-      case 13: epilogue_row_period<6, true>(args, taddr, row_valid, m, nb); return;
+      case 10:
+        if (estage)
+          epilogue_row_period_staged<5, false>(args, taddr, row_valid, m, nb, estage);
+        else
+          epilogue_row_period<5, false>(args, taddr, row_valid, m, nb);
+        return;
+      case 11:
+        if (estage)
+          epilogue_row_period_staged<5, true>(args, taddr, row_valid, m, nb, estage);
+        else
+          epilogue_row_period<5, true>(args, taddr, row_valid, m, nb);
+        return;
+      case 12:
+        if (estage)
+          epilogue_row_period_staged<6, false>(args, taddr, row_valid, m, nb, estage);
+        else
+          epilogue_row_period<6, false>(args, taddr, row_valid, m, nb);
+        return;
+      case 13:
+        if (estage)
+          epilogue_row_period_staged<6, true>(args, taddr, row_valid, m, nb, estage);
+        else
+          epilogue_row_period<6, true>(args, taddr, row_valid, m, nb);
+        return;
       case 14: epilogue_row_spec<7, false>(args, taddr, row_valid, m, nb); return;
       case 15: epilogue_row_spec<7, true>(args, taddr, row_valid, m, nb); return;
       case 16: epilogue_row_spec<8, false>(args, taddr, row_valid, m, nb); return;
@@ -1196,28 +1301,44 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
           }
         }
       };
-      long long ntile = first_tile;
-      int nj = 0;
       auto advance = [&](long long &tile, int &j) {
         if (++j == args.nck) {
           j = 0;
           tile += tile_step;
         }
       };
-      if (ntile < total_tiles) gather(ntile, nj, 0);
-      ptx::cp_async_commit();
-      long long ctile = ntile;
-      advance(ntile, nj);
-      for (long long k = 0; ctile < total_tiles; ++k) {
-        if (ntile < total_tiles) gather(ntile, nj, static_cast<int>((k + 1) & 1));
+      // Packed staging is a ring of D = gdepth slots: item k is gathered
+      // into slot k mod D, D - 1 items before it is widened. Each iteration
+      // commits exactly one cp.async group (empty past the last item), so
+      // waiting until at most D - 1 groups are pending means item k landed.
+      // A thread reads back only the rows it gathered itself, so refilling
+      // the slot it finished with one item earlier needs no barrier.
+      const int D = args.gdepth;
+      long long gtile = first_tile;  // issue side
+      int gj = 0, gslot = 0;
+      auto issue = [&]() {
+        if (gtile < total_tiles) gather(gtile, gj, gslot);
         ptx::cp_async_commit();
-        ptx::cp_async_wait<1>();  // item k of this thread's rows has landed
+        advance(gtile, gj);
+        if (++gslot == D) gslot = 0;
+      };
+      for (int d = 0; d + 1 < D; ++d) issue();
+      long long ctile = first_tile;  // widening side
+      int cj = 0, cslot = 0;
+      for (long long k = 0; ctile < total_tiles; ++k) {
+        issue();
+        if (D == 4)
+          ptx::cp_async_wait<3>();
+        else if (D == 3)
+          ptx::cp_async_wait<2>();
+        else
+          ptx::cp_async_wait<1>();  // item k of this thread's rows has landed
         const int hb = static_cast<int>(k & 1);
         if (k >= 2 && !wait_lane0(opempty(hb), static_cast<uint32_t>(((k >> 1) - 1) & 1))) {
           ok = false;
           break;
         }
-        const uint8_t *stg = sG + hb * args.g_stride;
+        const uint8_t *stg = sG + cslot * args.g_stride;
         for (int hr = t; hr < halo_rows; hr += kProdThreads) {
           if (voff(hr) < 0) continue;  // a row no tap reads
           W cur[WC];
@@ -1227,8 +1348,8 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         ptx::fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) ptx::mbar_arrive(opfull(hb));
-        ctile = ntile;
-        advance(ntile, nj);
+        advance(ctile, cj);
+        if (++cslot == D) cslot = 0;
       }
       ptx::cp_async_wait<0>();
     } else {
@@ -1329,6 +1450,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     // set `set` its half `set`. Warp w reads the TMEM lanes of quadrant w % 4.
     const int quad = warp & 3;
     const int set = (warp - kFirstEpiWarp) / 4;
+    uint32_t *const estage =
+        args.e_stage ? reinterpret_cast<uint32_t *>(smem + args.off_e) + (warp - kFirstEpiWarp) * 32 * kEpiPitch
+                     : nullptr;
     const int row = quad * 32 + lane;
     constexpr int kTileStep = HV == 2 ? 1 : 2;
     long long i = HV == 2 ? 0 : set;
@@ -1371,7 +1495,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       }
       const uint32_t taddr = tmem_base + static_cast<uint32_t>((acc_i * HV + (HV == 2 ? set : 0)) * args.mma_n) +
                              (static_cast<uint32_t>(quad * 32) << 16);
-      epilogue_row(args, taddr, valid && !warm, m, nb);
+      epilogue_row(args, taddr, valid && !warm, m, nb, estage);
       if (warm) {
         warm = false;
         continue;

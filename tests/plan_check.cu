@@ -37,7 +37,7 @@ samd_status conv2d_nchw(const samd_conv_desc *, samd_fmt, const void *, samd_fmt
 
 int main() {
   using namespace samd;
-  long long n = 0, bad = 0, halo = 0, seg = 0, fp8 = 0, res = 0, unsup = 0, hv2 = 0, win = 0;
+  long long n = 0, bad = 0, halo = 0, seg = 0, fp8 = 0, res = 0, unsup = 0, hv2 = 0, win = 0, deep = 0, estg = 0;
   const int Cs[] = {1, 3, 16, 24, 64, 96, 128, 256, 512, 1024};
   const int Ks[] = {1, 16, 40, 64, 96, 128, 256, 300, 512, 1024};
   const int HWs[] = {1, 2, 7, 14, 28, 56, 224};
@@ -55,7 +55,7 @@ int main() {
                       samd_conv_desc d{2, C, hw, hw, K, rs, rs, st, rs / 2, SAMD_NHWC};
                       samd_fmt fa{(uint8_t)ba, (uint8_t)sa, 0, (uint8_t)wb};
                       samd_fmt fw{(uint8_t)bw, (uint8_t)sw, 0, (uint8_t)wb};
-                      for (int fob : {0, 4, 6}) {
+                      for (int fob : {0, 3, 4, 6}) {
                         samd_fmt fo{(uint8_t)fob, 0, 0, 32};
                         conv::Plan p;
                         const samd_status s = conv::make_plan(&d, fa, fw, fo, p);
@@ -70,8 +70,12 @@ int main() {
                           ++halo;
                           if (p.nseg > 1) ++seg;
                           const int maxrow = (d.R - 1) * p.row_step + (d.S - 1) + 128 * p.hv - 1;
+                          const int srow = (p.WC * wb / 8 + 15) / 16 * 16;
                           ok = ok && maxrow < p.nseg * p.seg_rows &&
-                               p.nseg * p.seg_rows * static_cast<long long>(p.row_bytes) <= p.op_stride;
+                               p.nseg * p.seg_rows * static_cast<long long>(p.row_bytes) <= p.op_stride &&
+                               p.gdepth >= 2 && p.gdepth <= 4 &&
+                               static_cast<long long>(p.nseg) * p.seg_rows * srow <= p.g_stride;
+                          if (p.gdepth == 4) ++deep;
                         } else {
                           // gather staging: a producer group's ring of kGatherDepth x 128 rows
                           const int chunk_bytes = p.WC * wb / 8;
@@ -87,13 +91,17 @@ int main() {
                         if (p.b_resident) ++res;
                         if (p.hv == 2) ++hv2;
                         ok = ok && p.tmem_cols <= 512 && 2 * p.hv * p.mma_n <= static_cast<int>(p.tmem_cols);
+                        if (p.e_stage) {
+                          ++estg;
+                          ok = ok && (fob == 3 || fob == 5 || fob == 6) && p.off_e + conv::kEpiStageBytes <= p.off_bar;
+                        }
                         if (!ok && ++bad < 10)
                           printf("BAD C%d K%d hw%d rs%d st%d a%d%d w%d%d wb%d fo%d: smem %zu stages %d sta %d\n", C, K,
                                  hw, rs, st, ba, sa, bw, sw, wb, fob, p.smem_bytes, p.stages, p.stages_a);
                       }
                     }
   printf("plans %lld, bad %lld, unsupported %lld, halo %lld (segmented %lld), e4m3 %lld, resident %lld, "
-         "two-half %lld, window gather %lld\n",
-         n, bad, unsup, halo, seg, fp8, res, hv2, win);
+         "two-half %lld, window gather %lld, staging depth 4 %lld, staged epilogue %lld\n",
+         n, bad, unsup, halo, seg, fp8, res, hv2, win, deep, estg);
   return bad != 0;
 }
