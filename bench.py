@@ -44,6 +44,10 @@ def parse_args():
     ap.add_argument("--impl", default="samd", choices=["samd", "reference"])
     ap.add_argument("--workload", default="sweep", choices=["sweep", "vgg16", "resnet50", "conv1x"])
     ap.add_argument("--no-packed-ops", action="store_true")
+    ap.add_argument("--profile-ops", action="store_true",
+                    help="launch each packed op once at 2^28 lanes (b = 1, 4, 8; pack, unpack, the five elementwise "
+                         "ops) and the VGG-16 block-1 max-pool, after one untimed warm-up launch of each, and exit: "
+                         "the command ncu captures for the packed ops' DRAM counters")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
@@ -228,7 +232,9 @@ def workload_config(args, layers):
     desc = {
         "sweep": "3x3 conv N8 C64->64 56x56 pad1 stride1; act=weight=out width b in 1..8, signs uu/us/su/ss "
                  "(32 layers), int32 acc requantized to packed b-bit; 32-bit words",
-        "vgg16": "VGG-16 13 conv layers 224x224 batch16, u4 act x s4 wt -> u4 (pools excluded from timing)",
+        "vgg16": "VGG-16 13 conv layers 224x224 batch16, u4 act x s4 wt -> u4, chained: each layer reads the "
+                 "previous one's packed output, with the 4 2x2 max-pools between blocks in the timed step (fused "
+                 "into the conv epilogue for conv4, conv7 and conv10; standalone after conv2)",
         "resnet50": "ResNet-50 v1.5 stage convs (52) batch64, u6 act x s2 wt -> u6",
         "conv1x": "3x3 conv N1 C16->16 32x32, u4 x s4, 64-bit words",
     }[args.workload]
@@ -248,29 +254,126 @@ def workload_config(args, layers):
 
 # ---- the samd arm ------------------------------------------------------------------------
 
-def build_layers(layers, dev):
+def build_layers(layers, dev, chain=False):
+    """Packed inputs, prepared weights and output buffers of every layer.
+    With chain=True (VGG-16 as one network) only the first layer gets a
+    synthetic input; every other layer reads the previous layer's packed
+    output, or the 2x2 max-pool of it where the layer is marked pool_after
+    (the pool's output buffer is the entry's "pooled")."""
     import torch
 
     from paper_1809_10572_gb300 import samd, synth, workloads
 
     built = []
+    prev = None
     for i, layer in enumerate(layers):
         s = layer.shape
         fa = samd.fmt(layer.ba, layer.sa, 0, layer.word_bits)
         fw = samd.fmt(layer.bw, layer.sw, 0, layer.word_bits)
         fo = samd.fmt(layer.bo, layer.so, 0, layer.word_bits)
-        a = synth.lanes_t(synth.seed_for("bench", i), (s.N * s.H * s.W, s.C), layer.ba, layer.sa, device=dev)
-        a_w = samd.pack(synth.to_bytes_t(a), fa)
-        del a
+        if chain and prev is not None:
+            a_w = prev
+        else:
+            a = synth.lanes_t(synth.seed_for("bench", i), (s.N * s.H * s.W, s.C), layer.ba, layer.sa, device=dev)
+            a_w = samd.pack(synth.to_bytes_t(a), fa)
+            del a
         w = synth.lanes_t(synth.seed_for("benchw", i), (s.K * s.R * s.S, s.C), layer.bw, layer.sw, device=dev)
         w_w = samd.pack(synth.to_bytes_t(w), fw)
         conv = samd.PreparedConv(w_w, s, fa, fw, fo)
         _, out = conv.outputs(want_acc=False)
         shift = workloads.harness_shift(layer.ba, layer.bw, layer.bo, s.C * s.R * s.S)
         opb = samd.samd_conv2d_operand_bits(s.desc(), fa, fw)  # 8: e4m3 operands, 16: fp16
-        built.append({"layer": layer, "conv": conv, "act": a_w, "out": out, "shift": shift, "operand_bits": opb})
+        pooled, fused = None, False
+        if chain and layer.pool_after:
+            pooled = samd.empty_words(fo, s.N * (s.Ho // 2) * (s.Wo // 2), s.K, dev)
+            # the pool fused into the convolution's epilogue where the kernel
+            # supports it (samd_conv2d_prepared_pool2x2), else a second launch
+            fused = conv.pool2x2_supported()
+        built.append({"layer": layer, "conv": conv, "act": a_w, "out": out, "shift": shift, "operand_bits": opb,
+                      "fo": fo, "pooled": pooled, "fused_pool": fused})
+        prev = pooled if pooled is not None else out
     torch.cuda.synchronize()
     return built
+
+
+def _graph_time(fn, stream, reps=7):
+    """Median device time of fn's launches, captured once into a CUDA graph
+    and replayed (no host launch cost in the measurement)."""
+    import torch
+
+    with torch.cuda.stream(stream):
+        fn(stream)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        fn(torch.cuda.current_stream())
+    ts = []
+    for _ in range(reps):
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        g.replay()
+        s1.record(stream)
+        s1.synchronize()
+        ts.append(s0.elapsed_time(s1) * 1e-3)
+    return statistics.median(ts)
+
+
+def choose_pool_forms(built, stream):
+    """For each layer whose 2x2 max-pool the kernel can fuse, time the fused
+    call against the convolution followed by samd_maxpool2x2 (each alone, in
+    a CUDA graph) and keep the faster; returns the measured times (the two
+    forms give the same words, tests/test_gpu_pool.py)."""
+    from paper_1809_10572_gb300 import samd
+
+    forms = {}
+    for b in built:
+        if not b["fused_pool"]:
+            continue
+        s = b["layer"].shape
+
+        def fused(st, b=b):
+            b["conv"].pool2x2(b["act"], b["pooled"], b["shift"], stream=st)
+
+        def two(st, b=b, s=s):
+            b["conv"](b["act"], None, b["out"], b["shift"], stream=st)
+            samd.samd_maxpool2x2(b["fo"], b["out"], b["pooled"], s.N, s.K, s.Ho, s.Wo, stream=st)
+
+        tf, t2 = _graph_time(fused, stream), _graph_time(two, stream)
+        b["fused_pool"] = tf < t2
+        forms[b["layer"].name] = {"fused_us": tf * 1e6, "conv_then_pool_us": t2 * 1e6,
+                                  "chosen": "fused" if tf < t2 else "conv then pool"}
+    return forms
+
+
+def unique_bytes(built):
+    """Bytes of the distinct device tensors of a built workload."""
+    seen, total = set(), 0
+    for b in built:
+        for t in (b["act"], b["out"], b["conv"].prepared, b.get("pooled")):
+            if t is not None and t.data_ptr() not in seen:
+                seen.add(t.data_ptr())
+                total += t.numel() * t.element_size()
+    return total
+
+
+def launches_per_step(built):
+    return sum(1 + (1 if b.get("pooled") is not None and not b.get("fused_pool") else 0) for b in built)
+
+
+def run_chain(bs, stream):
+    """The layers of a chained network in order on one stream: each
+    convolution, then the 2x2 max-pool of its output where the network has
+    one (fused into the convolution where the kernel supports it)."""
+    from paper_1809_10572_gb300 import samd
+
+    for b in bs:
+        if b["fused_pool"]:
+            b["conv"].pool2x2(b["act"], b["pooled"], b["shift"], stream=stream)
+            continue
+        b["conv"](b["act"], None, b["out"], b["shift"], stream=stream)
+        if b["pooled"] is not None:
+            s = b["layer"].shape
+            samd.samd_maxpool2x2(b["fo"], b["out"], b["pooled"], s.N, s.K, s.Ho, s.Wo, stream=stream)
 
 
 def time_packed_ops(dev, flush):
@@ -379,6 +482,46 @@ def time_nchw_widemul(dev):
     return out
 
 
+def profile_ops():
+    """Each packed op once at 2^28 lanes for b = 1, 4, 8 (unsigned, 32-bit
+    words), then the 2x2 max-pool of VGG-16 block 1 (N16 224x224 C64 u4). The
+    first round of launches is a warm-up; the second is the one profiled
+    (ncu -s <launches of one round>). Prints the order of the launches."""
+    import torch
+
+    from paper_1809_10572_gb300 import samd, synth, workloads
+
+    dev = torch.device("cuda", 0)
+    samd.load()
+    n = workloads.ELEMENTWISE_N
+    calls = []
+    for b in (1, 4, 8):
+        f = samd.fmt(b, False)
+        xb = synth.to_bytes_t(synth.lanes_t(synth.seed_for("ewx", b, False), (n,), b, False, device=dev))
+        xw = samd.pack(xb, f)
+        yw = samd.pack(synth.to_bytes_t(synth.lanes_t(synth.seed_for("ewy", b, False, 0), (n,), b, False,
+                                                      device=dev)), f)
+        out = torch.empty_like(xw)
+        ub = torch.empty_like(xb)
+        calls.append((f"pack b{b}", lambda f=f, xb=xb, out=out: samd.samd_pack(f, xb, out, 1, n)))
+        calls.append((f"unpack b{b}", lambda f=f, xw=xw, ub=ub: samd.samd_unpack(f, xw, ub, 1, n)))
+        for op in workloads.ELEMENTWISE_OPS:
+            binary = op in ("add", "sub", "mul")
+            calls.append((f"{op} b{b}", lambda f=f, op=op, xw=xw, yw=yw, out=out, binary=binary: samd.samd_elementwise(
+                op, f, xw, yw if binary else None, f, out, n, 1 if op == "requant" else 0, 0)))
+    f4 = samd.fmt(4, False)
+    N, C, H, W = 16, 64, 224, 224
+    pin = samd.pack(synth.to_bytes_t(synth.lanes_t(5, (N * H * W, C), 4, False, device=dev)), f4)
+    pout = samd.empty_words(f4, N * H * W // 4, C, dev)
+    calls.append(("maxpool2x2 N16 C64 224x224 u4", lambda: samd.samd_maxpool2x2(f4, pin, pout, N, C, H, W)))
+    for rnd in range(2):
+        for name, fn in calls:
+            fn()
+        torch.cuda.synchronize()
+    print(json.dumps({"profile_ops": [name for name, _ in calls], "launches_per_round": len(calls)}), flush=True)
+    return 0
+
+
 def csrc_digest():
     """sha256 over the kernel sources (file names and contents)."""
     h = hashlib.sha256()
@@ -420,7 +563,9 @@ def run_samd(args, layers):
     # the sweep's 32 small layers run concurrently: each keeps to a few SMs
     tpc = args.tiles_per_cta or (8 if args.workload == "sweep" else 4)
     samd.samd_conv2d_set_min_tiles_per_cta(tpc)
-    built = build_layers(layers, dev)
+    chain = args.workload == "vgg16"  # one network: each layer reads the previous one's (pooled) output
+    built = build_layers(layers, dev, chain)
+    pool_forms = choose_pool_forms(built, torch.cuda.Stream(device=dev)) if chain else {}
     step_macs = workloads.total_macs(layers)
     # Between timed steps no step may find its data in L2. The step works on
     # one of R independent sets of inputs, prepared weights and outputs, the
@@ -428,10 +573,12 @@ def run_samd(args, layers):
     # when a set comes round again, more than an L2's worth of other data has
     # passed through since. (--l2 flush keeps one set and flushes L2 instead;
     # the line reports that number too.)
-    set_bytes = sum(t.numel() * t.element_size() for b in built
-                    for t in (b["act"], b["out"], b["conv"].prepared))
+    set_bytes = unique_bytes(built)
     n_sets = max(1, -(-2 * L2_BYTES // set_bytes)) if args.l2 == "rotate" else 1
-    sets = [built] + [build_layers(layers, dev) for _ in range(n_sets - 1)]
+    sets = [built] + [build_layers(layers, dev, chain) for _ in range(n_sets - 1)]
+    for bs in sets[1:]:  # the same choice in every set
+        for b, b0 in zip(bs, built):
+            b["fused_pool"] = b0["fused_pool"]
     flush_w = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     flush_r = torch.ones(L2_FLUSH_BYTES // 8, dtype=torch.int64, device=dev)
 
@@ -446,6 +593,9 @@ def run_samd(args, layers):
     side = [torch.cuda.Stream(device=dev) for _ in range(max(1, args.streams))]
 
     def step_calls(main, bs):
+        if chain:
+            run_chain(bs, main)
+            return
         # the layers of the workload are independent: fan them out over the
         # side streams and join them back into `main`
         for sd in side:
@@ -568,8 +718,12 @@ def run_samd(args, layers):
                 "frac_vs_nominal_ratio": achieved_tflops / (2.0 * step_macs / sum(
                     2.0 * b["layer"].macs / ((2.0 if b["operand_bits"] == 8 else 1.0) * bf16_peak * 1e12)
                     for b in built) / 1e12),
-                "note": "achieved = 2 x direct-conv MACs of the step / step time (all launches are the conv kernel); "
-                        "frac_vs_nominal_ratio takes e4m3 at 2 x the bf16 peak instead"}
+                "note": ("achieved = 2 x direct-conv MACs of the step / step time (the step's "
+                         f"{launches_per_step(built) - len(built)} standalone max-pool launches and "
+                         f"{sum(1 for b in built if b.get('fused_pool'))} fused pool epilogues included, so "
+                         "achieved is understated); " if chain else
+                         "achieved = 2 x direct-conv MACs of the step / step time (all launches are the conv "
+                         "kernel); ") + "frac_vs_nominal_ratio takes e4m3 at 2 x the bf16 peak instead"}
 
     line = {
         "metric": METRIC, "value": value, "unit": "MAC/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
@@ -578,7 +732,7 @@ def run_samd(args, layers):
         "data": "synthetic",
         "config": workload_config(args, layers), "l2_sets": l2_note, "value_l2_flushed": value_flushed,
         "wall_s_timed_region": wall,
-        "gpu_launches": args.steps * len(built),
+        "gpu_launches": args.steps * launches_per_step(built),
         "roofline": roofline,
     }
     if args.workload == "sweep":
@@ -587,6 +741,8 @@ def run_samd(args, layers):
             per_bits.setdefault(name.split("_")[0], []).append(v)
         line["by_bits_mac_s"] = {k: statistics.mean(v) for k, v in per_bits.items()}
     line["by_layer_mac_s"] = by_layer
+    if pool_forms:
+        line["pool_forms"] = pool_forms
 
     # int8 tensor-core peak (for the metric's "fraction of int8 TC peak")
     if rank == 0:
@@ -596,7 +752,7 @@ def run_samd(args, layers):
 
     # e2e: the same step through the C ABI from pinned host buffers
     if not args.no_e2e:
-        line["e2e"] = measure_e2e(built, step_macs, args, dev, ws, d)
+        line["e2e"] = measure_e2e(built, step_macs, args, dev, ws, d, chain)
 
     if rank == 0 and not args.no_packed_ops:
         ops = time_packed_ops(dev, flush)
@@ -675,13 +831,29 @@ def measure_int8_peak(dev):
                 tops = 2 * macs.value / (ms.value * 1e-3) / 1e12
                 best = tops if best is None else max(best, tops)
         res["mma_sync_s8_tops"] = best
+        # the binary MMA (m16n8k256 b1, AND + popcount): the bit-plane form of
+        # a 1-2-bit convolution takes b^2 of its products per multiply-add
+        lib.samd_peak_bmma_b1.argtypes = lib.samd_peak_imma_s8.argtypes
+        lib.samd_peak_bmma_b1.restype = ctypes.c_int
+        bbest = None
+        for per_sm in (2, 4, 8):
+            ms, ops = ctypes.c_float(0), ctypes.c_double(0)
+            rc = lib.samd_peak_bmma_b1(sms * per_sm, 4096, scratch.data_ptr(), ctypes.byref(ms), ctypes.byref(ops))
+            if rc == 0 and ms.value > 0:
+                r = ops.value / (ms.value * 1e-3)
+                bbest = r if bbest is None else max(bbest, r)
+        res["mma_sync_b1_products_per_s"] = bbest
+        if bbest:
+            res["bitplane_mac_s"] = {"b1": bbest, "b2": bbest / 4}
     except Exception as e:  # noqa: BLE001
         res["mma_sync_s8_tops"] = None
         res["mma_sync_error"] = f"{type(e).__name__}: {e}"
     vals = [v for v in (res.get("int_mm_tops"), res.get("mma_sync_s8_tops")) if v]
     res["tops"] = max(vals) if vals else None
     res["how"] = ("best of torch._int_mm int8 8192^3 (best of 5) and a hand-written mma.sync m16n8k32 s8 loop on "
-                  "register operands (2, 4, 8 blocks of 256 threads per SM, 4096 x 8 MMAs per warp)")
+                  "register operands (2, 4, 8 blocks of 256 threads per SM, 4096 x 8 MMAs per warp); "
+                  "mma_sync_b1_products_per_s: the same loop on mma.sync m16n8k256 b1 AND+popc; bitplane_mac_s: "
+                  "the multiply-add rate of a bit-plane convolution built on it (b^2 binary products per b-bit MAC)")
     return res
 
 
@@ -703,14 +875,19 @@ def measure_e4m3_peak(dev):
         return {"tflops": None, "how": f"torch._scaled_mm unavailable: {type(e).__name__}: {e}"}
 
 
-def measure_e2e(built, step_macs, args, dev, ws, d):
+def measure_e2e(built, step_macs, args, dev, ws, d, chain=False):
     import torch
 
-    host_in = [torch.empty(b["act"].shape, dtype=b["act"].dtype, pin_memory=True) for b in built]
-    host_out = [torch.empty(b["out"].shape, dtype=b["out"].dtype, pin_memory=True) for b in built]
-    for h, b in zip(host_in, built):
+    # a chained network copies in the first layer's input and copies out the
+    # last layer's output; independent layers copy each layer's own
+    ends = [built[0]] if chain else built
+    host_in = [torch.empty(b["act"].shape, dtype=b["act"].dtype, pin_memory=True) for b in ends]
+    last = built[-1]["pooled"] if (chain and built[-1]["pooled"] is not None) else built[-1]["out"]
+    host_out = ([torch.empty(last.shape, dtype=last.dtype, pin_memory=True)] if chain else
+                [torch.empty(b["out"].shape, dtype=b["out"].dtype, pin_memory=True) for b in built])
+    for h, b in zip(host_in, ends):
         h.copy_(b["act"])
-    dev_in = [torch.empty_like(b["act"]) for b in built]
+    dev_in = [b["act"] for b in ends] if chain else [torch.empty_like(b["act"]) for b in built]
     h2d = sum(t.numel() * t.element_size() for t in host_in)
     d2h = sum(t.numel() * t.element_size() for t in host_out)
     # each layer's copy in, convolution and copy out run in order on one of
@@ -722,6 +899,12 @@ def measure_e2e(built, step_macs, args, dev, ws, d):
     samd.samd_conv2d_set_min_tiles_per_cta(tpc)
 
     def calls(main):
+        if chain:
+            with torch.cuda.stream(main):
+                dev_in[0].copy_(host_in[0], non_blocking=True)
+                run_chain(built, main)
+                host_out[0].copy_(last, non_blocking=True)
+            return
         for st in streams:
             st.wait_stream(main)
         for i, (b, hi, di, ho) in enumerate(zip(built, host_in, dev_in, host_out)):
@@ -766,10 +949,12 @@ def measure_e2e(built, step_macs, args, dev, ws, d):
     el_eager = timed(step_eager)
     if samd.samd_device_status() != 0:
         raise RuntimeError("a kernel recorded a timeout")
+    how = ("one CUDA graph per step: pinned H2D of the network's packed input, the chained layers and pools, "
+           "pinned D2H of the last packed output; host replays and waits each step" if chain else
+           "one CUDA graph per step: per layer, on one of the step's streams, pinned H2D of its packed input, "
+           "samd_conv2d_prepared, pinned D2H of its packed output; host replays and waits each step")
     return {"value": step_macs * args.steps * ws / el, "unit": "MAC/s", "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h,
-            "how": "one CUDA graph per step: per layer, on one of the step's streams, pinned H2D of its packed input, "
-                   "samd_conv2d_prepared, pinned D2H of its packed output; host replays and waits each step",
+            "d2h_bytes_per_step": d2h, "how": how,
             "eager_value": step_macs * args.steps * ws / el_eager,
             "eager_how": "the same calls issued from Python every step (no graph): host-bound"}
 
@@ -780,6 +965,8 @@ def main():
         os.environ["CUDA_DEVICE_MAX_CONNECTIONS"] = str(args.connections)
     from paper_1809_10572_gb300 import workloads
 
+    if args.profile_ops:
+        return profile_ops()
     layers = workloads.WORKLOADS[args.workload]()
     if args.layers:
         idx = [int(t) for t in args.layers.split(",")]

@@ -241,6 +241,31 @@ SAMD_API samd_status samd_conv2d_noalloc(const samd_conv_desc *desc, samd_fmt fa
                                          samd_stream_t stream);
 
 /*
+ * samd_conv2d_prepared_pool2x2: samd_conv2d_prepared followed by the 2x2
+ * max-pool of samd_maxpool2x2, in one kernel (the paper has no pooling; the
+ * VGG-16 stack pools after conv2, conv4, conv7, conv10 and conv13). The
+ * convolution's packed rows never reach memory: pooled_out receives
+ * N*(Ho/2)*(Wo/2) rows of K elements packed along K in format fo, row
+ * (n, i, j) holding the lane-wise max over the 2x2 window at output rows
+ * 2i, 2i+1 and columns 2j, 2j+1 of clamp_fo(floor(acc / 2^shift)) -- the
+ * same words samd_conv2d_prepared and then samd_maxpool2x2 produce.
+ * `prepared` is what samd_conv2d_prepare wrote for the same desc, fa, fw and
+ * fo. Supported shapes (samd_conv2d_pool2x2_supported, host-only, tells;
+ * else SAMD_EUNSUP and nothing is launched): NHWC, stride 1, Ho and Wo even,
+ * 2 * (W + 2 * pad) <= 256 (a tile of 256 positions holds whole pairs of
+ * padded image rows), fo of 1, 2, 4 or 8 bits in 32-bit words without
+ * spacers, and a layer the kernel runs as halo tiles of two halves with
+ * room for the tile's packed rows in shared memory. pooled_out: 16-byte
+ * aligned, caller-owned.
+ */
+SAMD_API samd_status samd_conv2d_prepared_pool2x2(const samd_conv_desc *desc, samd_fmt fa, const void *act,
+                                                  samd_fmt fw, const void *prepared, size_t prepared_bytes,
+                                                  samd_fmt fo, void *pooled_out, int shift, samd_stream_t stream);
+/* 1 if samd_conv2d_prepared_pool2x2 supports this shape and these formats,
+ * else 0 (invalid arguments included). Host-only; no GPU needed. */
+SAMD_API int samd_conv2d_pool2x2_supported(const samd_conv_desc *desc, samd_fmt fa, samd_fmt fw, samd_fmt fo);
+
+/*
  * samd_maxpool2x2: lane-wise max over 2x2 windows with stride 2 (used
  * between the VGG-16 blocks; not in the paper). Layout SAMD_NHWC: in is
  * N*H*W rows of C elements packed along C, out is N*(H/2)*(W/2) rows.

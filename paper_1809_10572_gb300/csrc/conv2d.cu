@@ -192,7 +192,7 @@ struct Plan {
   int hv;         // tile of hv halves of 128 output positions
   int row_bytes;  // operand row: 64 (e4m3) or 128 (fp16) bytes
   int wpr, words_total, La, WC, nchunks, Kpad, NBc, n_mma, mma_n, split, nblocks, stages, Ho, Wo, gather_vec;
-  int gather_win;  // 1x1 gather through 16-byte windows (AGather::issue_win)
+  int gather_win;  // gather through 16-byte windows (AGather::issue_win); chunks = (channel chunk, tap)
   int g_row;       // gather staging row pitch in bytes
   int halo, Hv, Wp, nck, taps;
   int nseg, seg_rows, seg_used, row_step;  // halo geometry (see ConvArgs)
@@ -200,6 +200,7 @@ struct Plan {
   int stages_a, b_resident;
   int gdepth;  // HALO: packed staging slots (items gathered gdepth - 1 ahead of the widening)
   int e_stage; // kEpiStageBytes at off_e stage the epilogue's 3/5/6-bit packed rows
+  int pool, pool_rows, pool_nw, pool_pitch, pool_tpi;  // fused 2x2 max-pool (ConvArgs::pool)
   long long M;
   long long bound;  // R*S*C * max|a| * max|w|: no accumulator exceeds it
   uint32_t tmem_cols;
@@ -213,13 +214,14 @@ long long max_abs(samd_fmt f) { return f.is_signed ? (1LL << (f.bits - 1)) : ((1
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 constexpr int kMaxHaloRows = 1024;
+constexpr int kHaloGatherDepth = 2;  // packed staging slots of the halo producers (2..4)
 // minimum 128-pixel tiles per CTA of a launch (samd_conv2d_set_min_tiles_per_cta)
 std::atomic<int> g_min_tiles_per_cta{4};
 
 // Tiling, reduction order, operand type and exactness mode for one
 // convolution. fo.bits == 0 means no packed output. Returns SAMD_EUNSUP when
 // no mode keeps every accumulator below 2^24.
-samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fmt fo, Plan &p) {
+samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fmt fo, Plan &p, bool pool = false) {
   p.La = lanes_per_word(fa);
   if (p.La == 0) return SAMD_EINVAL;
   const long long taps = static_cast<long long>(d->R) * d->S * d->C;
@@ -263,11 +265,15 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
   const int srow = (chunk_bytes + 15) / 16 * 16;  // Staging::kRowBytes
   const int vec = chunk_bytes % 16 == 0 ? 16 : (chunk_bytes % 8 == 0 ? 8 : wb);
   p.gather_vec = (p.wpr % p.WC == 0) && ((static_cast<long long>(p.wpr) * wb) % vec == 0) ? 1 : 0;
-  // A 1x1 layer whose chunks are not whole 16-byte vectors copies each
+  // A gather layer whose chunks are not whole 16-byte vectors copies each
   // chunk through the 16-byte-aligned window around it: one more 16-byte
   // piece than the chunk, and an odd number of pieces per staging row, so
   // that a quarter-warp's 16-byte accesses to eight rows hit distinct banks.
-  p.gather_win = (!(p.gather_vec && vec == 16) && d->R == 1 && d->S == 1) ? 1 : 0;
+  // Its chunks are (channel chunk, tap) pairs, each inside one pixel (as in
+  // the halo path), so that a chunk is one contiguous run of a pixel's words
+  // however the pixel's word count divides into chunks (strided 3x3 layers
+  // whose chunks would otherwise straddle pixels and be copied word by word).
+  p.gather_win = (p.gather_vec && vec == 16) ? 0 : 1;
   int win_pieces = srow / 16 + 1;
   if (win_pieces % 2 == 0) ++win_pieces;
   const int grow = p.gather_win ? win_pieces * 16 : srow;
@@ -276,10 +282,10 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
   const size_t bst = p.b_bytes;
   const size_t e_bytes = 0;  // the epilogue packs in registers
   // mbarriers: full_b and empty_b per weight stage, opfull and opempty per
-  // operand stage, two accumulator pairs and the drain barrier; then the
-  // TMEM address word
+  // operand stage, two accumulator pairs, the drain barrier and two
+  // epilogue group barriers; then the TMEM address word
   auto bar_bytes = [](int stages, int op_stages) {
-    return round_up(static_cast<size_t>(2 * stages + 2 * op_stages + 5) * 8 + 4, 16);
+    return round_up(static_cast<size_t>(2 * stages + 2 * op_stages + 7) * 8 + 4, 16);
   };
   const size_t kBudget = 224 * 1024;  // below the 227 KB opt-in limit minus static shared memory
   auto finish = [&](size_t op_bytes, size_t g_bytes, int op_stages) {
@@ -291,6 +297,10 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
   };
   p.taps = d->R * d->S;
   p.nck = (p.wpr + p.WC - 1) / p.WC;
+  if (p.gather_win) {  // (channel chunk, tap) chunks
+    p.nchunks = p.nck * p.taps;
+    p.Kpad = p.nchunks * BK;
+  }
   p.Hv = d->H + 2 * d->pad;
   p.Wp = d->W + 2 * d->pad;
   const int nchunks_gather = p.nchunks;
@@ -333,12 +343,14 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
       const size_t stage_g = round_up(static_cast<size_t>(halo_rows) * srow, 16);
       const int ntiles_b = p.nck * p.taps;
       if (halo_rows > kMaxHaloRows || waste > 1.16) return false;
-      // The deepest packed staging ring (4, 3 or 2 items) that fits: with
-      // depth D the gathers run D - 1 items ahead of the widening, which
-      // hides the global-memory latency behind D - 1 items of MMA work.
+      // The packed staging ring: with depth D the gathers run D - 1 items
+      // ahead of the widening. Depth 2 is used: per-role timelines show the
+      // halo producers finishing a tile's operands microseconds before its
+      // MMAs start, and the sweep step measured 6% slower at depth 4 (the
+      // kernel takes depths up to 4).
       size_t fixed = 0;
       bool res = false;
-      int depth = 4;
+      int depth = kHaloGatherDepth;
       for (; depth >= 2; --depth) {
         fixed = 2 * halo_bytes + depth * stage_g + e_bytes + 1024;
         if (fixed + 2 * bst + bar_bytes(2, 2) > kBudget) continue;
@@ -398,15 +410,69 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
       placed = place(halo, hv, need_res != 0);
     }
   if (!placed) return SAMD_EUNSUP;  // operand tiles do not fit (not reached for N <= 256)
+  // Fused 2x2 max-pool: tiles must hold whole pairs of padded image rows,
+  // 2 Wp <= 128 hv. Halo layers are placed again with the most tile halves
+  // that allow it (the weight layout of a halo layer does not depend on the
+  // halves or on residency, so the same prepared weights serve both forms).
+  if (pool) {
+    if (!p.halo) return SAMD_EUNSUP;
+    placed = false;
+    for (int hv = 2; hv >= 1 && !placed; --hv) {
+      if ((hv == 2 && !two) || 2 * p.Wp > BM * hv) continue;
+      for (int need_res = 1; need_res >= 0 && !placed; --need_res) placed = place(true, hv, need_res != 0);
+    }
+    if (!placed) return SAMD_EUNSUP;
+  }
   // 3-, 5- and 6-bit packed outputs (32-bit words, no spacer) stage their
-  // rows in shared memory when that fits beside the placement chosen above
-  // (which it never changes), so that stores are contiguous within a row.
+  // rows in shared memory when a channel block's row holds at least one
+  // whole packing period (lcm(32, L) channels: 160 for L = 5 or 10, 96 for
+  // L = 6) and the buffer fits beside the placement chosen above (which it
+  // never changes), so that stores are contiguous within a row. Shorter rows
+  // (64 channels: 7 to 13 words) measured faster stored directly.
   p.e_stage = 0;
+  const int period_ch = fo.bits == 5 ? 96 : 160;
   if ((fo.bits == 3 || fo.bits == 5 || fo.bits == 6) && fo.spacer == 0 && fo.word_bits == 32 &&
-      p.smem_bytes + round_up(kEpiStageBytes, 16) <= kBudget) {
+      p.NBc >= period_ch && p.smem_bytes + round_up(kEpiStageBytes, 16) <= kBudget) {
     p.e_stage = 1;
     p.off_bar = static_cast<uint32_t>(round_up(p.off_e + kEpiStageBytes, 16));
     p.smem_bytes = 1024 + p.off_bar + bar_bytes(p.stages, p.halo ? 2 : p.stages_a);
+  }
+  // Fused 2x2 max-pool (placed above): even output sizes, outputs of 1, 2, 4
+  // or 8 bits in 32-bit words. A tile is q = 128 hv / (2 Wp) row pairs of
+  // one image; its packed rows are staged in 256 rows of pool_pitch words
+  // (odd, so that the epilogue threads' word stores spread over the banks)
+  // after the other regions: one buffer of 256 rows for two-half tiles, one
+  // of 128 rows per epilogue set for one-half tiles.
+  p.pool = 0;
+  if (pool) {
+    const int Ho = p.Ho, Wo = p.Wo;
+    if (!p.halo || d->stride != 1 || (Ho & 1) || (Wo & 1) || Ho < 2 || 2 * p.Wp > BM * p.hv || fo.spacer != 0 ||
+        fo.word_bits != 32 || (fo.bits != 1 && fo.bits != 2 && fo.bits != 4 && fo.bits != 8))
+      return SAMD_EUNSUP;
+    int q = (BM * p.hv) / (2 * p.Wp);
+    if (q > Ho / 2) q = Ho / 2;
+    const int Lo = 32 / fo.bits;
+    p.pool_rows = 2 * q;
+    p.pool_tpi = (Ho / 2 + q - 1) / q;
+    p.pool_nw = (p.NBc + Lo - 1) / Lo;
+    p.pool_pitch = p.pool_nw | 1;
+    const size_t pool_bytes = static_cast<size_t>(2 * BM) * p.pool_pitch * 4;
+    if (p.e_stage) return SAMD_EUNSUP;  // not reached: e_stage is for 3/5/6-bit outputs
+    // the buffer goes after the packed staging ring, made shallower if need
+    // be (the ring's depth does not change the weight layout)
+    int depth = p.gdepth;
+    size_t off_e = 0;
+    for (; depth >= 2; --depth) {
+      off_e = round_up(p.off_g + static_cast<size_t>(depth) * p.g_stride, 16);
+      if (1024 + round_up(off_e + pool_bytes, 16) + bar_bytes(p.stages, 2) <= kBudget) break;
+    }
+    if (depth < 2) return SAMD_EUNSUP;
+    p.pool = 1;
+    p.gdepth = depth;
+    p.grid_m = static_cast<long long>(d->N) * p.pool_tpi;
+    p.off_e = static_cast<uint32_t>(off_e);
+    p.off_bar = static_cast<uint32_t>(round_up(off_e + pool_bytes, 16));
+    p.smem_bytes = 1024 + p.off_bar + bar_bytes(p.stages, 2);
   }
   uint32_t cols = 32;
   while (cols < static_cast<uint32_t>(2 * p.hv * p.mma_n)) cols <<= 1;  // two accumulators of hv halves
@@ -422,13 +488,15 @@ samd_fmt none_fmt() { return samd_fmt{0, 0, 0, 0}; }
 bool layout_ok(const Plan &p) {
   const size_t NO = p.halo ? 2 : static_cast<size_t>(p.stages_a);
   const size_t op_bytes = NO * p.op_stride;
-  const size_t bars = (2 * static_cast<size_t>(p.stages) + 2 * NO + 5) * 8 + 4;
+  const size_t bars = (2 * static_cast<size_t>(p.stages) + 2 * NO + 7) * 8 + 4;
   return p.stages >= 1 && NO >= 2 && op_bytes <= p.off_b &&
          p.off_b + static_cast<size_t>(p.stages) * p.b_bytes <= p.off_g && p.off_g + static_cast<size_t>(p.halo ? p.gdepth : 2) * p.g_stride <= p.off_e &&
          p.off_e <= p.off_bar && 1023 + p.off_bar + bars <= p.smem_bytes && p.op_stride % 1024 == 0 &&
          p.off_b % 1024 == 0 && p.b_bytes % 1024 == 0 && p.off_bar % 8 == 0 && 2 * p.hv * p.mma_n <= 512 &&
          (p.hv == 1 || p.hv == 2) && (!p.halo || (p.gdepth >= 2 && p.gdepth <= 4)) &&
-         (!p.e_stage || p.off_e + kEpiStageBytes <= p.off_bar);
+         (!p.e_stage || p.off_e + kEpiStageBytes <= p.off_bar) &&
+         (!p.pool || (p.halo && 2 * p.Wp <= BM * p.hv && !p.e_stage && p.pool_pitch >= p.pool_nw &&
+                      p.off_e + static_cast<size_t>(2 * BM) * p.pool_pitch * 4 <= p.off_bar));
 }
 
 // Device address of a __device__ symbol in the current context, looked up
@@ -490,6 +558,11 @@ int conv2d_operand_bits(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw) {
   return p.fp8 ? 8 : 16;
 }
 
+int conv2d_pool_supported(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fmt fo) {
+  conv::Plan p;
+  return (conv::make_plan(d, fa, fw, fo, p, true) == SAMD_OK && conv::layout_ok(p)) ? 1 : 0;
+}
+
 samd_status conv2d_check(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw) {
   conv::Plan p;
   return conv::make_plan(d, fa, fw, conv::none_fmt(), p);
@@ -523,7 +596,7 @@ samd_status conv2d_prepare(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, co
   wa.mma_n = p.mma_n;
   wa.NBc = p.NBc;
   wa.split = p.split;
-  wa.halo = p.halo;
+  wa.halo = p.halo || p.gather_win;  // reduction order (channel chunk, tap, position)
   wa.taps = p.taps;
   wa.rows_total = static_cast<long long>(p.nblocks) * p.mma_n;
   const long long total = wa.rows_total * wa.Kpad;
@@ -544,10 +617,14 @@ samd_status conv2d_prepare(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, co
 
 samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const void *act, const void *prepared,
                        size_t prepared_bytes, int32_t *acc_out, samd_fmt fo, void *packed_out, int shift,
-                       cudaStream_t s) {
+                       cudaStream_t s, void *pooled_out) {
   using namespace conv;
   Plan p;
-  samd_status st = make_plan(d, fa, fw, fo, p);
+  // pooled_out: the 2x2 max-pool of the packed output is the only output
+  const bool pool = pooled_out != nullptr;
+  if (pool && (acc_out || packed_out)) return SAMD_EINVAL;
+  if (pool) packed_out = pooled_out;
+  samd_status st = make_plan(d, fa, fw, fo, p, pool);
   if (st != SAMD_OK) return st;
   if (prepared_bytes < p.ws_bytes) return SAMD_ESHAPE;
   if (p.M == 0) return SAMD_OK;
@@ -651,6 +728,11 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   a.gdepth = p.gdepth;
   a.off_e = p.off_e;
   a.e_stage = p.e_stage;
+  a.pool = p.pool;
+  a.pool_rows = p.pool ? p.pool_rows : 0;
+  a.pool_nw = p.pool ? p.pool_nw : 0;
+  a.pool_pitch = p.pool ? p.pool_pitch : 0;
+  a.fd_tpi = make_fastdiv(static_cast<uint32_t>(p.pool ? p.pool_tpi : 1));
   a.off_bar = p.off_bar;
   // A small layer gives each CTA at least T reference tiles of work (T from
   // samd_conv2d_set_min_tiles_per_cta; a reference tile is 128 positions of
@@ -661,7 +743,11 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   // spread over more SMs.
   const long long total_tiles = p.grid_m * p.nblocks;
   const long long ref_work = static_cast<long long>(g_min_tiles_per_cta.load(std::memory_order_relaxed)) * 9 * 64;
-  const long long tile_work = static_cast<long long>(p.hv) * p.nchunks * p.mma_n;
+  long long tile_work = static_cast<long long>(p.hv) * p.nchunks * p.mma_n;
+  // A gather tile with a short reduction (1x1 layers over few channels) is
+  // bound by widening its lanes and packing its outputs, not by its MMAs:
+  // it counts as at least one reference tile per half.
+  if (!p.halo && tile_work < static_cast<long long>(p.hv) * 9 * 64) tile_work = static_cast<long long>(p.hv) * 9 * 64;
   long long min_tiles = ref_work / tile_work;
   if (min_tiles < 1) min_tiles = 1;
   long long ctas = (total_tiles + min_tiles - 1) / min_tiles;

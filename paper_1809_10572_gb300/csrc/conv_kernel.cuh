@@ -159,7 +159,7 @@ struct ConvArgs {
   long long grid_m; // 128-position tiles along the output
   int nblocks;      // channel blocks
   int gather_vec;   // AGather::vec
-  int gather_win;   // AGather::issue_win (1x1 layers whose chunks are not aligned vectors)
+  int gather_win;   // AGather::issue_win (chunks that are not aligned 16-byte vectors); chunk = (channel chunk, tap)
   int g_row;        // GATHER staging row pitch in bytes
   int gdepth;       // HALO: packed staging slots; gathers run gdepth - 1 items ahead
   long long act_bytes;  // bytes of the activation tensor (the windows stop at its end)
@@ -189,7 +189,26 @@ struct ConvArgs {
   uint32_t op_stride;  // one halo buffer or one A tile
   uint32_t off_b, b_bytes, off_g, g_stride, off_e, off_bar;
   int e_stage;  // 1: kEpiStageBytes at off_e stage the 3/5/6-bit packed rows (epilogue_row_period_staged)
+  // Fused 2x2 max-pool (pool = 1; halo layers): tile mt is pool_rows output
+  // rows (pool_rows / 2 row pairs) of one image from an even row on, at
+  // virtual position img * Hv * Wp + g * pool_rows * Wp (img = mt / tiles
+  // per image, g its remainder). The epilogue warps that drain a tile pack
+  // its rows into the pool_pitch-word rows of their buffer at off_e (pool_nw
+  // words of the channel block per row) and write only the lane-wise maxima
+  // of the 2x2 windows, rows of (N, Ho / 2, Wo / 2) pixels, to packed_out.
+  int pool, pool_rows, pool_nw, pool_pitch;
+  FastDiv fd_tpi;  // tiles per image
 };
+
+// First position, in the padded virtual grid N x Hv x Wp, of tile mt of a
+// halo layer (tiles of bmt consecutive positions, or pooled tiles of whole
+// row pairs).
+__device__ __forceinline__ uint32_t tile_first_pos(const ConvArgs &args, uint32_t mt, int bmt) {
+  if (!args.pool) return mt * static_cast<uint32_t>(bmt);
+  const uint32_t img = fdiv(mt, args.fd_tpi);
+  const uint32_t g = mt - img * args.fd_tpi.d;
+  return img * args.fd_plane.d + g * static_cast<uint32_t>(args.pool_rows * args.Wp);
+}
 
 __device__ __forceinline__ uint32_t hsub2_bits(uint32_t a, uint32_t b) {
   uint32_t r;
@@ -424,7 +443,7 @@ __device__ __forceinline__ void load_window(const uint8_t *row, int o4, int nw, 
 template <typename W, int WC>
 struct AGather {
   const W *act;
-  int H, W_, wpr, S, stride, pad, words_total;
+  int H, W_, wpr, S, stride, pad, words_total, taps;
   int n, oh, ow;
   bool row_valid;
   bool vec;  // every chunk lies inside one pixel at a kVec-aligned offset
@@ -461,18 +480,21 @@ struct AGather {
     }
   }
 
-  // 1x1 layers (one tap): the chunk's bytes are copied as the 16-byte pieces
+  // Chunks that are not whole 16-byte vectors (issue_win): chunk c is
+  // channel chunk j = c / taps of the pixel at tap c % taps, the words
+  // [j WC, min((j + 1) WC, wpr)) of that pixel, copied as the 16-byte pieces
   // of the aligned window around them, so that every copy is 16 bytes wide
   // whatever the pixel's alignment. Pieces past the chunk are zero-filled;
   // a piece that reaches past the end of the activation tensor (act_end)
   // copies only the bytes before it. Returns the chunk's offset into the
   // staged row in 32-bit units (load_window). act is 16-byte aligned.
   __device__ __forceinline__ int issue_win(int chunk, uint32_t dst, uintptr_t act_end) const {
-    const int kw0 = chunk * WC;
-    const int nw = words_total - kw0 < WC ? words_total - kw0 : WC;
+    const int j = chunk / taps;
+    const int wi = j * WC;
+    const int nw = wpr - wi < WC ? wpr - wi : WC;
     bool valid;
-    const W *px = pixel(0, valid);
-    const uintptr_t a = valid ? reinterpret_cast<uintptr_t>(px + kw0) : reinterpret_cast<uintptr_t>(act);
+    const W *px = pixel(chunk - j * taps, valid);
+    const uintptr_t a = valid ? reinterpret_cast<uintptr_t>(px + wi) : reinterpret_cast<uintptr_t>(act);
     const uintptr_t a0 = a & ~static_cast<uintptr_t>(15);
     const uintptr_t end = a + static_cast<uintptr_t>(nw) * sizeof(W);
 #pragma unroll
@@ -951,6 +973,115 @@ __device__ __forceinline__ void epilogue_row(const ConvArgs &args, uint32_t tadd
   }
 }
 
+// The epilogue warps' meeting point of a pooled tile: every warp of the
+// tile's group arrives on `bar` once its part of the step is done, then
+// waits, bounded, for the phase; false if the wait gave up.
+__device__ __forceinline__ bool epi_group_sync(uint32_t bar, uint32_t &phase, volatile int *status) {
+  __syncwarp();
+  bool ok = true;
+  if ((threadIdx.x & 31) == 0) {
+    ptx::mbar_arrive(bar);
+    ok = ptx::mbar_wait_bounded(bar, phase & 1u, status, kWaitLimitNs);
+  }
+  ++phase;
+  ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+  __syncwarp();
+  return ok;
+}
+
+// Epilogue of one pooled tile for output lanes of OB = 1, 2, 4 or 8 bits
+// (32-bit words, no spacers), called by each warp of the tile's group of
+// gw warps (gi = this warp's index in it) for its 32 rows:
+// requantize and pack the row (tile row trow) into the pool buffer, free the
+// accumulator, meet the other epilogue warps, then write the lane-wise max of
+// every 2x2 window of the tile's row pairs (the maximum commutes with the
+// monotone requantize, so this is the pool of the requantized output), and
+// meet again before the buffer is reused. False if a wait gave up.
+template <int OB, bool OS>
+__device__ __noinline__ bool epilogue_pool_tile(const ConvArgs &args, uint32_t taddr, int trow, uint32_t mt, int nb,
+                                                uint32_t *pbuf, uint32_t acc_empty, uint32_t group_bar,
+                                                uint32_t &phase, volatile int *status, int gw, int gi) {
+  constexpr int LH = 32 / OB;  // lanes per word
+  constexpr int NH = 32 / LH;  // words per 32 channels
+  constexpr int32_t lo = OS ? -(1 << (OB - 1)) : 0, hi = OS ? (1 << (OB - 1)) - 1 : (1 << OB) - 1;
+  constexpr int32_t blo = kMagicBits + lo, bhi = kMagicBits + hi;
+  constexpr uint32_t omask = (1u << OB) - 1;
+  constexpr uint32_t bias_sum = [] {
+    uint32_t b = 0;
+    for (int l = 0; l < LH; ++l) b += static_cast<uint32_t>(kMagicBits) << (l * OB);
+    return b;
+  }();
+  const int ch0 = nb * args.NBc;
+  const int nvalid = args.K - ch0 < args.NBc ? args.K - ch0 : args.NBc;
+  const int nw = (nvalid + LH - 1) / LH;  // this block's words of a row (<= pool_nw; fewer in a last, partial block)
+  const int pitch = args.pool_pitch;
+  const float scale = args.out_scale;
+  uint32_t *prow = pbuf + trow * pitch;
+  for (int col = 0; col < nvalid; col += 32) {
+    uint32_t r[32];
+    ptx::tmem_ld_32x32b_x32(taddr + col, r);
+    ptx::tmem_wait_ld();
+    const int cnt = nvalid - col < 32 ? nvalid - col : 32;
+#pragma unroll
+    for (int j = 0; j < NH; ++j) {
+      uint32_t w = 0;
+#pragma unroll
+      for (int l = 0; l < LH; ++l) {
+        int32_t t = floor_scaled_biased(__uint_as_float(r[j * LH + l]), scale);
+        t = t < blo ? blo : (t > bhi ? bhi : t);
+        if (j * LH + l >= cnt) t = kMagicBits;  // lanes past the block's channels stay zero
+        if constexpr (OS)
+          w |= (static_cast<uint32_t>(t) & omask) << (l * OB);
+        else
+          w += static_cast<uint32_t>(t) << (l * OB);
+      }
+      const int wi = col / LH + j;
+      if (wi < nw) prow[wi] = OS ? w : w - bias_sum;
+    }
+  }
+  ptx::tc_fence_before();
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) ptx::mbar_arrive(acc_empty);
+  if (!epi_group_sync(group_bar, phase, status)) return false;
+  // the 2x2 windows of this tile's row pairs
+  const uint32_t img = fdiv(mt, args.fd_tpi);
+  const int g = static_cast<int>(mt - img * args.fd_tpi.d);
+  const int Ho2 = args.Ho / 2, Wo2 = args.Wo / 2, q = args.pool_rows / 2;
+  const int q_here = Ho2 - g * q < q ? Ho2 - g * q : q;
+  const int total = q_here * Wo2 * nw;
+  const uint32_t flip = OS ? LaneMsb<uint32_t, OB>::kValue : 0u;
+  uint32_t *out = static_cast<uint32_t *>(args.packed_out) + ch0 / LH;
+  const int Wp = args.Wp;
+  for (int idx = 32 * gi + static_cast<int>(threadIdx.x & 31); idx < total; idx += 32 * gw) {
+    const int pix = idx / nw, w = idx - (idx / nw) * nw;
+    const int i = pix / Wo2, j = pix - (pix / Wo2) * Wo2;
+    const uint32_t *b0 = pbuf + (2 * i * Wp + 2 * j) * pitch + w;
+    const uint32_t top = swar_lane_max<uint32_t, OB>(b0[0], b0[pitch], flip);
+    const uint32_t bot = swar_lane_max<uint32_t, OB>(b0[Wp * pitch], b0[(Wp + 1) * pitch], flip);
+    const long long orow = (static_cast<long long>(img) * Ho2 + g * q + i) * Wo2 + j;
+    out[orow * args.out_wpr + w] = swar_lane_max<uint32_t, OB>(top, bot, flip);
+  }
+  return epi_group_sync(group_bar, phase, status);
+}
+
+__device__ __forceinline__ bool epilogue_pool_dispatch(const ConvArgs &args, uint32_t taddr, int trow, uint32_t mt,
+                                                       int nb, uint32_t *pbuf, uint32_t acc_empty, uint32_t group_bar,
+                                                       uint32_t &phase, volatile int *status, int gw, int gi) {
+#define SAMD_POOL_TILE(OB, OS) \
+  epilogue_pool_tile<OB, OS>(args, taddr, trow, mt, nb, pbuf, acc_empty, group_bar, phase, status, gw, gi)
+  switch (args.out_bits * 2 + (args.out_signed ? 1 : 0)) {
+    case 2: return SAMD_POOL_TILE(1, false);
+    case 3: return SAMD_POOL_TILE(1, true);
+    case 4: return SAMD_POOL_TILE(2, false);
+    case 5: return SAMD_POOL_TILE(2, true);
+    case 8: return SAMD_POOL_TILE(4, false);
+    case 9: return SAMD_POOL_TILE(4, true);
+    case 16: return SAMD_POOL_TILE(8, false);
+    default: return SAMD_POOL_TILE(8, true);
+  }
+#undef SAMD_POOL_TILE
+}
+
 // One MMA.
 template <bool FP8>
 __device__ __forceinline__ void mma_op(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
@@ -1067,9 +1198,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
   uint8_t *sB = smem + args.off_b;
   uint8_t *sG = smem + args.off_g;  // packed staging
   uint64_t *bars = reinterpret_cast<uint64_t *>(smem + args.off_bar);
-  // barriers: full_b[STB] empty_b[STB] opfull[NO] opempty[NO] accfull[2] accempty[2] drain
+  // barriers: full_b[STB] empty_b[STB] opfull[NO] opempty[NO] accfull[2] accempty[2] drain group[2]
   const int NO = HALO ? 2 : args.stages_a;
-  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 2 * STB + 2 * NO + 5);
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 2 * STB + 2 * NO + 7);
   auto full_b = [&](int s) { return ptx::smem_addr(bars + s); };
   auto empty_b = [&](int s) { return ptx::smem_addr(bars + STB + s); };
   auto opfull = [&](int s) { return ptx::smem_addr(bars + 2 * STB + s); };
@@ -1077,6 +1208,9 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
   auto accfull = [&](int a) { return ptx::smem_addr(bars + 2 * STB + 2 * NO + a); };
   auto accempty = [&](int a) { return ptx::smem_addr(bars + 2 * STB + 2 * NO + 2 + a); };
   const uint32_t drain_bar = ptx::smem_addr(bars + 2 * STB + 2 * NO + 4);
+  // the epilogue warps of a pooled tile: all eight (two-half tiles), or the
+  // four of epilogue set g (one-half tiles, group_bar(g))
+  auto group_bar = [&](int g) { return ptx::smem_addr(bars + 2 * STB + 2 * NO + 5 + g); };
 
   volatile int *status = args.status;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -1100,6 +1234,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       ptx::mbar_init(accempty(a), HV == 2 ? kEpiWarps : kEpiWarps / 2);  // the warps that drain accumulator a
     }
     ptx::mbar_init(drain_bar, 1);
+    for (int g = 0; g < 2; ++g) ptx::mbar_init(group_bar(g), HV == 2 ? kEpiWarps : kEpiWarps / 2);
     ptx::fence_barrier_init();
   }
   __syncwarp();  // every warp reaches the barrier converged (bar.sync counts whole warps)
@@ -1189,7 +1324,10 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
           ok = false;
           break;
         }
-        int words = (HALO ? args.wpr : args.words_total) - j * WC;
+        // words of the packed chunk: channel chunk j (halo) or j / taps
+        // (window gather) of a pixel, else words j WC.. of the whole reduction
+        int words = HALO ? args.wpr - j * WC
+                         : (args.gather_win ? args.wpr - (j / args.taps) * WC : args.words_total - j * WC);
         if (words > WC) words = WC;
         int npos = words * U::L;
         if (npos > BK) npos = BK;  // FULL: the last word's lanes past 64 are padding
@@ -1272,7 +1410,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       // items k = (tile i, channel chunk j), in the MMA's order
       auto gather = [&](long long tile, int j, int slot) {
         const uint32_t mt = static_cast<uint32_t>(tile) - fdiv(static_cast<uint32_t>(tile), args.fd_gm) * args.fd_gm.d;
-        const uint32_t v0 = mt * BMT;
+        const uint32_t v0 = tile_first_pos(args, mt, BMT);
         const uint32_t dst0 = ptx::smem_addr(sG + slot * args.g_stride);
         for (int hr = t; hr < halo_rows; hr += kProdThreads) {
           const int off = voff(hr);
@@ -1368,6 +1506,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       g.stride = args.stride;
       g.pad = args.pad;
       g.words_total = args.words_total;
+      g.taps = args.taps;
       g.vec = args.gather_vec != 0;
       auto set_tile = [&](long long tile) {
         const uint32_t tl = static_cast<uint32_t>(tile);
@@ -1423,7 +1562,8 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         const uint8_t *srow = sG + grp * (kGatherDepth * kSlotBytes) + slot * kSlotBytes + (t % BM) * g_row;
         if (win) {
           const int chunk = static_cast<int>(k % nchunks);
-          const int nw = args.words_total - chunk * WC < WC ? args.words_total - chunk * WC : WC;
+          const int wi = (chunk / args.taps) * WC;
+          const int nw = args.wpr - wi < WC ? args.wpr - wi : WC;
           load_window<W, WC>(srow, static_cast<int>((o4s >> (2 * slot)) & 3u), nw, cur);
         } else {
           load_staged<W, WC>(srow, cur);
@@ -1462,7 +1602,45 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     // instructions are fetched while the first tile is being computed rather
     // than after it.
     bool warm = true;
-    for (long long tile = first_tile + (HV == 2 ? 0 : set) * tile_step; tile < total_tiles;) {
+    bool pooled = false;
+    if constexpr (HALO) {
+      if (args.pool) {
+        // pooled tiles (no warm-up pass): two-half tiles are drained and
+        // pooled by all eight epilogue warps, one-half tiles by the four of
+        // the set that drains them (alternate tiles, own buffer and barrier)
+        pooled = true;
+        constexpr int gw = HV == 2 ? kEpiWarps : kEpiWarps / 2;
+        const int gi = HV == 2 ? warp - kFirstEpiWarp : warp - kFirstEpiWarp - 4 * set;
+        uint32_t *const pbuf = reinterpret_cast<uint32_t *>(smem + args.off_e) + (HV == 2 ? 0 : set * BM * args.pool_pitch);
+        const uint32_t gbar = group_bar(HV == 2 ? 0 : set);
+        constexpr int kStep = HV == 2 ? 1 : 2;
+        uint32_t gphase = 0;
+        long long ip = HV == 2 ? 0 : set;
+        for (long long tile = first_tile + (HV == 2 ? 0 : set) * tile_step; tile < total_tiles;
+             tile += kStep * tile_step, ip += kStep) {
+          const int acc_i = HV == 2 ? static_cast<int>(ip & 1) : set;
+          bool w_ok = true;
+          if (lane == 0)
+            w_ok = ptx::mbar_wait_bounded(accfull(acc_i), static_cast<uint32_t>((ip >> 1) & 1), status, kWaitLimitNs);
+          if (!__shfl_sync(0xffffffffu, w_ok ? 1 : 0, 0)) {
+            ok = false;
+            break;
+          }
+          ptx::tc_fence_after();
+          const uint32_t tl = static_cast<uint32_t>(tile);
+          const uint32_t nbu = fdiv(tl, args.fd_gm);
+          const uint32_t mt = tl - nbu * args.fd_gm.d;
+          const uint32_t taddr = tmem_base + static_cast<uint32_t>((acc_i * HV + (HV == 2 ? set : 0)) * args.mma_n) +
+                                 (static_cast<uint32_t>(quad * 32) << 16);
+          if (!epilogue_pool_dispatch(args, taddr, (HV == 2 ? set * BM : 0) + row, mt, static_cast<int>(nbu), pbuf,
+                                      accempty(acc_i), gbar, gphase, status, gw, gi)) {
+            ok = false;
+            break;
+          }
+        }
+      }
+    }
+    for (long long tile = first_tile + (HV == 2 ? 0 : set) * tile_step; !pooled && tile < total_tiles;) {
       const int acc_i = HV == 2 ? static_cast<int>(i & 1) : set;  // accumulator of this tile
       if (!warm) {
         bool w_ok = true;
@@ -1482,7 +1660,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       long long m;
       const int trow = (HV == 2 ? set * BM : 0) + row;  // row of the tile
       if (HALO) {
-        const uint32_t v = mt * BMT + trow;
+        const uint32_t v = tile_first_pos(args, mt, BMT) + trow;
         const uint32_t img = fdiv(v, args.fd_plane);
         const uint32_t rem = v - img * args.fd_plane.d;
         const uint32_t oh = fdiv(rem, args.fd_wp);

@@ -321,9 +321,11 @@ __device__ __forceinline__ W field_sub(W a, W b, const FieldMasks<W> &f, bool is
 
 template <typename W>
 __device__ __forceinline__ W field_mul(W a, W b, const FieldMasks<W> &f, bool is_signed, bool sat) {
-  if (!sat && f.bits <= 2) {
+  if (!sat) {
     // Fig. 6 shift-and-add over the fields: step j adds a << j where bit j
-    // of the lane of b is set, cut at the top of the lane's data bits
+    // of the lane of b is set, cut at the top of the lane's data bits; bits
+    // steps of a few word operations each, against L lanes of extract,
+    // multiply and insert
     W acc = 0;
     for (int j = 0; j < f.bits; ++j) {
       const W bit = b & (f.lsb << j);

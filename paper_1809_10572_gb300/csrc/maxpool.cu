@@ -17,24 +17,8 @@ namespace {
 constexpr int kThreads = 256;
 
 template <typename W, int BITS>
-struct PoolMasks {
-  static constexpr int L = WordTraits<W>::kBits / BITS;
-  static constexpr W msb() {
-    W m = 0;
-    for (int i = 0; i < L; ++i) m |= W(1) << (i * BITS + BITS - 1);
-    return m;
-  }
-  static constexpr W kMsb = msb();
-};
-
-template <typename W, int BITS>
 __device__ __forceinline__ W swar_max(W a, W b, W flip) {
-  constexpr W M = PoolMasks<W, BITS>::kMsb;
-  W x = a ^ flip, y = b ^ flip;                        // offset-binary for signed lanes
-  W d = ((x ^ y) & M) ^ ((x | M) - (y & ~M)) ^ M;       // lane-wise x - y
-  W lt = ((~x & y) | ((~x | y) & d)) & M;               // borrow out of the lane: x < y
-  W E = (lt - (lt >> (BITS - 1))) | lt;                 // whole lanes where x < y
-  return (b & E) | (a & ~E);
+  return swar_lane_max<W, BITS>(a, b, flip);
 }
 
 // Blocks loop over output rows (image n, row i); threads run over the row's
@@ -46,7 +30,7 @@ __global__ void __launch_bounds__(kThreads) maxpool_swar_kernel(const W *__restr
                                                                 int Wo, int H, int W_, int wpr, int is_signed, int rows) {
   const int upp = wpr / V;  // units per pixel
   const int units = Wo * upp;
-  const W flip = is_signed ? PoolMasks<W, BITS>::kMsb : W(0);
+  const W flip = is_signed ? LaneMsb<W, BITS>::kValue : W(0);
   for (int row = blockIdx.x; row < rows; row += gridDim.x) {  // row = n * Ho + i
   const int n = row / Ho, i = row - (row / Ho) * Ho;
   const W *top = in + (static_cast<long long>(n) * H + 2 * i) * W_ * wpr;

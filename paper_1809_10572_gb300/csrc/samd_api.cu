@@ -190,6 +190,26 @@ samd_status samd_conv2d_prepared(const samd_conv_desc *d, samd_fmt fa, const voi
                     reinterpret_cast<cudaStream_t>(stream));
 }
 
+samd_status samd_conv2d_prepared_pool2x2(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw,
+                                         const void *prepared, size_t prepared_bytes, samd_fmt fo, void *pooled_out,
+                                         int shift, samd_stream_t stream) {
+  if (!pooled_out || fo.bits == 0) return SAMD_EINVAL;
+  samd_status st = conv_common_checks(d, fa, fw, fo, shift);
+  if (st != SAMD_OK) return st;
+  if (d->layout != SAMD_NHWC) return SAMD_EUNSUP;
+  if (d->N == 0) return SAMD_OK;
+  if (!conv2d_pool_supported(d, fa, fw, fo)) return SAMD_EUNSUP;
+  if (!act || !prepared) return SAMD_EINVAL;
+  if (!aligned16(act) || !aligned16(prepared) || !aligned16(pooled_out)) return SAMD_EALIGN;
+  return conv2d_run(d, fa, fw, act, prepared, prepared_bytes, nullptr, fo, nullptr, shift,
+                    reinterpret_cast<cudaStream_t>(stream), pooled_out);
+}
+
+int samd_conv2d_pool2x2_supported(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fmt fo) {
+  if (!d || fo.bits == 0 || conv_common_checks(d, fa, fw, fo, 0) != SAMD_OK || d->layout != SAMD_NHWC) return 0;
+  return conv2d_pool_supported(d, fa, fw, fo);
+}
+
 samd_status samd_maxpool2x2(samd_fmt f, const void *in, void *out, int N, int C, int H, int W, samd_layout layout,
                             samd_stream_t stream) {
   if (!fmt_valid(f)) return SAMD_EINVAL;

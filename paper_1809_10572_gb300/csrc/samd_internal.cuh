@@ -114,6 +114,32 @@ __device__ __forceinline__ W field_max(W a, W b, const FieldMasks<W> &f, W flip)
   return (a & E) | (b & ~E & f.live);
 }
 
+// The top bit of every lane of a spacer-free word of BITS-bit lanes.
+template <typename W, int BITS>
+struct LaneMsb {
+  static constexpr W mask() {
+    W m = 0;
+    for (int i = 0; i < WordTraits<W>::kBits / BITS; ++i) m |= W(1) << (i * BITS + BITS - 1);
+    return m;
+  }
+  static constexpr W kValue = mask();
+};
+
+// Lane-wise max of two words of spacer-free BITS-bit lanes, flip = the msb
+// mask for signed lanes (offset binary orders like two's complement), else
+// 0. A lane-wise subtract with the lane MSBs as temporary spacers (section 3,
+// Fig. 5) gives each lane's borrow, i.e. x < y, which selects the larger
+// lane.
+template <typename W, int BITS>
+__device__ __forceinline__ W swar_lane_max(W a, W b, W flip) {
+  constexpr W M = LaneMsb<W, BITS>::kValue;
+  const W x = a ^ flip, y = b ^ flip;
+  const W d = ((x ^ y) & M) ^ ((x | M) - (y & ~M)) ^ M;  // lane-wise x - y
+  const W lt = ((~x & y) | ((~x | y) & d)) & M;          // borrow out of the lane: x < y
+  const W E = (lt - (lt >> (BITS - 1))) | lt;            // whole lanes where x < y
+  return (b & E) | (a & ~E);
+}
+
 }  // namespace samd
 
 // ---- launchers implemented in the kernel translation units ----------------
@@ -131,12 +157,13 @@ samd_status conv2d_prepare(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, co
                            void *prepared, size_t prepared_bytes, cudaStream_t s);
 samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const void *act, const void *prepared,
                        size_t prepared_bytes, int32_t *acc_out, samd_fmt fo, void *packed_out, int shift,
-                       cudaStream_t s);
+                       cudaStream_t s, void *pooled_out = nullptr);
 samd_status conv2d_nhwc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,
                         int32_t *acc_out, samd_fmt fo, void *packed_out, int shift, void *workspace,
                         size_t workspace_bytes, cudaStream_t s);
 size_t conv2d_workspace_size(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw);
 int conv2d_operand_bits(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw);
+int conv2d_pool_supported(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fmt fo);
 void conv2d_set_min_tiles_per_cta(int tiles);
 constexpr size_t kNoallocScratchBytes = size_t(8) << 20;  // static scratch of samd_conv2d_noalloc
 samd_status conv2d_noalloc(const samd_conv_desc *d, samd_fmt fa, const void *act, samd_fmt fw, const void *wt,

@@ -44,7 +44,7 @@ OPS = {"add": SAMD_ADD, "sub": SAMD_SUB, "mul": SAMD_MUL, "relu": SAMD_RELU, "re
 
 EXPORTED = ["samd_lanes_per_word", "samd_packed_words", "samd_pack", "samd_unpack", "samd_elementwise",
             "samd_conv2d", "samd_conv2d_workspace_size", "samd_conv2d_operand_bits", "samd_conv2d_set_min_tiles_per_cta", "samd_conv2d_prepare", "samd_conv2d_prepared",
-            "samd_conv2d_noalloc",
+            "samd_conv2d_noalloc", "samd_conv2d_prepared_pool2x2", "samd_conv2d_pool2x2_supported",
             "samd_maxpool2x2", "samd_device_status", "samd_selftest_wait_timeout", "samd_status_str", "samd_version"]
 FMT_NONE = (0, 0, 0, 0)
 
@@ -91,6 +91,11 @@ def load(build_if_missing: bool = True):
     lib.samd_conv2d_prepared.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, vp, samd_fmt, vp, sz, vp, samd_fmt, vp,
                                          i32, vp]
     lib.samd_conv2d_prepared.restype = i32
+    lib.samd_conv2d_prepared_pool2x2.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, vp, samd_fmt, vp, sz, samd_fmt,
+                                                 vp, i32, vp]
+    lib.samd_conv2d_prepared_pool2x2.restype = i32
+    lib.samd_conv2d_pool2x2_supported.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, samd_fmt, samd_fmt]
+    lib.samd_conv2d_pool2x2_supported.restype = i32
     lib.samd_conv2d_workspace_size.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, samd_fmt]
     lib.samd_conv2d_workspace_size.restype = sz
     lib.samd_conv2d_operand_bits.argtypes = [c.POINTER(samd_conv_desc), samd_fmt, samd_fmt]
@@ -217,6 +222,18 @@ def samd_conv2d_prepared(desc, fa, act, fw, prepared, acc_out, fo, packed_out, s
     nb = _nbytes(prepared) if prepared_bytes is None else prepared_bytes
     _check(load().samd_conv2d_prepared(ctypes.byref(desc), fa, _ptr(act), fw, _ptr(prepared), nb, _ptr(acc_out), fo,
                                        _ptr(packed_out), shift, _stream(stream)), "samd_conv2d_prepared")
+
+
+def samd_conv2d_prepared_pool2x2(desc, fa, act, fw, prepared, fo, pooled_out, shift, prepared_bytes=None,
+                                 stream=None):
+    nb = _nbytes(prepared) if prepared_bytes is None else prepared_bytes
+    _check(load().samd_conv2d_prepared_pool2x2(ctypes.byref(desc), fa, _ptr(act), fw, _ptr(prepared), nb, fo,
+                                               _ptr(pooled_out), shift, _stream(stream)),
+           "samd_conv2d_prepared_pool2x2")
+
+
+def samd_conv2d_pool2x2_supported(desc, fa, fw, fo) -> bool:
+    return bool(load().samd_conv2d_pool2x2_supported(ctypes.byref(desc), fa, fw, fo))
 
 
 def samd_maxpool2x2(f, inp, out, N, C, H, W, layout=SAMD_NHWC, stream=None):
@@ -351,6 +368,16 @@ class PreparedConv:
         samd_conv2d_prepared(self.shape.desc(), self.fa, act, self.fw, self.prepared, acc_out, self.fo, packed_out,
                              shift, stream=stream)
         return acc_out, packed_out
+
+    def pool2x2_supported(self) -> bool:
+        return self.fo is not None and samd_conv2d_pool2x2_supported(self.shape.desc(), self.fa, self.fw, self.fo)
+
+    def pool2x2(self, act, pooled_out, shift: int = 0, stream=None):
+        """The convolution with the 2x2 max-pool of its packed output fused
+        (samd_conv2d_prepared_pool2x2)."""
+        samd_conv2d_prepared_pool2x2(self.shape.desc(), self.fa, act, self.fw, self.prepared, self.fo, pooled_out,
+                                     shift, stream=stream)
+        return pooled_out
 
     def outputs(self, want_acc=True, want_packed=True, device="cuda"):
         s = self.shape

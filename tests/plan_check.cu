@@ -75,7 +75,7 @@ int main() {
                                p.nseg * p.seg_rows * static_cast<long long>(p.row_bytes) <= p.op_stride &&
                                p.gdepth >= 2 && p.gdepth <= 4 &&
                                static_cast<long long>(p.nseg) * p.seg_rows * srow <= p.g_stride;
-                          if (p.gdepth == 4) ++deep;
+                          if (p.gdepth == conv::kHaloGatherDepth) ++deep;
                         } else {
                           // gather staging: a producer group's ring of kGatherDepth x 128 rows
                           const int chunk_bytes = p.WC * wb / 8;
@@ -84,7 +84,9 @@ int main() {
                                p.g_stride >= static_cast<uint32_t>(conv::kGatherDepth * conv::BM * p.g_row);
                           if (p.gather_win) {
                             ++win;
-                            ok = ok && d.R == 1 && d.S == 1 && p.g_row >= srow + 16 && (p.g_row / 16) % 2 == 1;
+                            // (channel chunk, tap) chunks, each inside one pixel
+                            ok = ok && p.g_row >= srow + 16 && (p.g_row / 16) % 2 == 1 &&
+                                 p.nchunks == p.nck * p.taps && p.nck * p.WC >= p.wpr && (p.nck - 1) * p.WC < p.wpr;
                           }
                         }
                         if (p.fp8) ++fp8;
@@ -101,7 +103,7 @@ int main() {
                       }
                     }
   printf("plans %lld, bad %lld, unsupported %lld, halo %lld (segmented %lld), e4m3 %lld, resident %lld, "
-         "two-half %lld, window gather %lld, staging depth 4 %lld, staged epilogue %lld\n",
+         "two-half %lld, window gather %lld, staging at the chosen depth %lld, staged epilogue %lld\n",
          n, bad, unsup, halo, seg, fp8, res, hv2, win, deep, estg);
   return bad != 0;
 }

@@ -148,3 +148,26 @@ def test_min_tiles_per_cta_setting(lib):
     assert lib.samd_conv2d_set_min_tiles_per_cta(1025) == samd.SAMD_EINVAL
     assert lib.samd_conv2d_set_min_tiles_per_cta(8) == samd.SAMD_OK
     assert lib.samd_conv2d_set_min_tiles_per_cta(4) == samd.SAMD_OK  # the default again
+
+
+def test_fused_pool_support_query(lib):
+    # host-only: which layers samd_conv2d_prepared_pool2x2 runs (halo tiles
+    # holding whole pairs of padded rows, even outputs, 1/2/4/8-bit outputs
+    # in 32-bit words without spacers)
+    from paper_1809_10572_gb300 import workloads
+
+    fa, fw, u4 = samd.fmt(4, False), samd.fmt(4, True), samd.fmt(4, False)
+    got = {l.name: samd.samd_conv2d_pool2x2_supported(l.shape.desc(), fa, fw, u4)
+           for l in workloads.vgg16() if l.pool_after}
+    assert got == {"conv2": False, "conv4": True, "conv7": True, "conv10": True}  # conv2: 2 (224 + 2) > 256
+    s = samd.ConvShape(2, 64, 56, 56, 64)
+    assert samd.samd_conv2d_pool2x2_supported(s.desc(), fa, fw, u4)
+    for fo in (samd.fmt(1, False), samd.fmt(2, True), samd.fmt(8, True)):
+        assert samd.samd_conv2d_pool2x2_supported(s.desc(), fa, fw, fo)
+    for fo in (samd.fmt(3, False), samd.fmt(4, False, spacer=1), samd.fmt(4, False, word_bits=64),
+               samd.fmt(*samd.FMT_NONE)):
+        assert not samd.samd_conv2d_pool2x2_supported(s.desc(), fa, fw, fo)
+    for bad in (samd.ConvShape(2, 64, 56, 57, 64), samd.ConvShape(2, 64, 56, 56, 64, stride=2),
+                samd.ConvShape(2, 64, 8, 8, 64)):
+        assert not samd.samd_conv2d_pool2x2_supported(bad.desc(), fa, fw, u4)
+    assert not samd.samd_conv2d_pool2x2_supported(s.desc(samd.SAMD_NCHW), fa, fw, u4)

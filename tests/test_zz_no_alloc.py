@@ -46,13 +46,14 @@ def check_case(shape, ba, sa, bw, sw, fo, shift, seed, want_acc=True):
 def test_noalloc_matches_oracle_on_consecutive_calls(samd_lib):
     # calls in a row on the same static array: a larger layer first, then a
     # smaller one that reuses (and must fully rewrite) its start; a layer
-    # whose widened weights fill the array exactly (8 MiB, split weight
-    # digits: 2016 taps x 255 x 128 is past 2^24); an output with no int32
-    # accumulator; and the first layer again
+    # whose widened weights fill the array exactly (8 MiB: 1x1 over 2048
+    # channels to 960, split weight digits since 2048 x 255 x 128 is past
+    # 2^24, eight channel blocks of 2 x 128 rows x 2048 fp16 positions); an
+    # output with no int32 accumulator; and the first layer again
     cases = [
         (samd.ConvShape(2, 64, 14, 14, 96), 4, False, 4, True, samd.fmt(4, False), 6, 101, True),
         (samd.ConvShape(1, 24, 9, 7, 40), 6, True, 8, True, samd.fmt(6, True), 8, 202, True),
-        (samd.ConvShape(1, 224, 8, 8, 960), 8, False, 8, True, samd.fmt(8, False), 12, 303, True),
+        (samd.ConvShape(1, 2048, 2, 2, 960, R=1, S=1, pad=0), 8, False, 8, True, samd.fmt(8, False), 12, 303, True),
         (samd.ConvShape(2, 40, 7, 9, 72, R=1, S=1, pad=0), 6, False, 2, True, samd.fmt(6, False), 3, 404, False),
         (samd.ConvShape(1, 33, 5, 6, 20), 3, True, 5, False, None, 0, 606, True),  # int32 output only
         (samd.ConvShape(2, 64, 14, 14, 96), 4, False, 4, True, samd.fmt(4, False), 6, 505, True),
@@ -63,11 +64,10 @@ def test_noalloc_matches_oracle_on_consecutive_calls(samd_lib):
 
 
 def test_noalloc_rejects_layers_beyond_its_scratch(samd_lib):
-    # The limit applies to the widened weights of the call itself. 976 output
-    # channels of 3-bit lanes (10 per word) take channel blocks of 120: nine
-    # blocks, 9 MiB. (With no packed output the same layer takes eight blocks
-    # of 128 and fills the array exactly; samd_conv2d_workspace_size reports
-    # the larger need over every output format.)
+    # The limit applies to the widened weights of the call itself: 976
+    # output channels of 3-bit lanes (10 per word) take nine channel blocks
+    # of 120 over 36 chunks (four per pixel and tap), 10.6 MB; and a 3x3
+    # layer over 1024 channels to 1024, 11.8 MB.
     cases = [(samd.ConvShape(1, 224, 8, 8, 976), samd.fmt(8, False), samd.fmt(8, True), samd.fmt(3, False)),
              (samd.ConvShape(1, 1024, 4, 4, 1024), samd.fmt(4, False), samd.fmt(4, True), None)]
     for shape, fa, fw, fo in cases:
