@@ -307,12 +307,13 @@ def _graph_time(fn, stream, reps=7):
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, stream=stream):
         fn(torch.cuda.current_stream())
+    cur = torch.cuda.current_stream()  # replay() launches the graph here
     ts = []
     for _ in range(reps):
         s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        s0.record(stream)
+        s0.record(cur)
         g.replay()
-        s1.record(stream)
+        s1.record(cur)
         s1.synchronize()
         ts.append(s0.elapsed_time(s1) * 1e-3)
     return statistics.median(ts)

@@ -199,6 +199,7 @@ struct Plan {
   long long grid_m;                        // 128-position tiles along the output
   int stages_a, b_resident;
   int gdepth;  // HALO: packed staging slots (items gathered gdepth - 1 ahead of the widening)
+  int hbufs;   // HALO: widened halo buffers (2 or 3)
   int e_stage; // kEpiStageBytes at off_e stage the epilogue's 3/5/6-bit packed rows
   int pool, pool_rows, pool_nw, pool_pitch, pool_tpi;  // fused 2x2 max-pool (ConvArgs::pool)
   long long M;
@@ -312,6 +313,7 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
     p.hv = hv;
     p.halo = 0;
     p.gdepth = 2;
+    p.hbufs = 2;
     p.b_resident = 0;
     p.stages_a = 0;
     p.nseg = p.seg_rows = p.seg_used = p.row_step = 0;
@@ -348,18 +350,32 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
       // halo producers finishing a tile's operands microseconds before its
       // MMAs start, and the sweep step measured 6% slower at depth 4 (the
       // kernel takes depths up to 4).
+      // Widened halo buffers: the producers widen item k into buffer
+      // k mod hbufs once the MMAs of item k - hbufs are done. fp16 layers
+      // take three when their weights stay resident as well. (A 6-bit sweep
+      // layer's tiles came 2.9 -> 2.2 us apart with three buffers and
+      // streamed weights, but the layer as a whole, four tiles per CTA, ran
+      // 10-20% slower without resident weights; e4m3 layers, whose halo is
+      // half as large and cheaper to widen, showed no gain.)
       size_t fixed = 0;
       bool res = false;
-      int depth = kHaloGatherDepth;
-      for (; depth >= 2; --depth) {
-        fixed = 2 * halo_bytes + depth * stage_g + e_bytes + 1024;
-        if (fixed + 2 * bst + bar_bytes(2, 2) > kBudget) continue;
-        res = p.nblocks == 1 && fixed + ntiles_b * bst + bar_bytes(ntiles_b, 2) <= kBudget;
-        if (need_resident && !res) continue;
-        break;
+      int depth = kHaloGatherDepth, hbufs = 2;
+      auto fits = [&](int nb, int dp, bool want_res) {
+        fixed = nb * halo_bytes + dp * stage_g + e_bytes + 1024;
+        if (fixed + 2 * bst + bar_bytes(2, nb) > kBudget) return false;
+        res = p.nblocks == 1 && fixed + ntiles_b * bst + bar_bytes(ntiles_b, nb) <= kBudget;
+        return !(want_res && !res);
+      };
+      bool ok3 = !p.fp8 && fits(3, depth, true);
+      if (ok3) {
+        hbufs = 3;
+      } else {
+        for (; depth >= 2; --depth)
+          if (fits(2, depth, need_resident)) break;
+        if (depth < 2) return false;
       }
-      if (depth < 2) return false;
       p.gdepth = depth;
+      p.hbufs = hbufs;
       p.halo = 1;
       p.nchunks = ntiles_b;
       p.Kpad = ntiles_b * BK;
@@ -368,12 +384,12 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
         p.b_resident = 1;
         p.stages = ntiles_b;
       } else {
-        long long st = static_cast<long long>((kBudget - fixed - bar_bytes(8, 2)) / bst);
+        long long st = static_cast<long long>((kBudget - fixed - bar_bytes(8, hbufs)) / bst);
         p.stages = static_cast<int>(st > 8 ? 8 : st);
       }
       p.op_stride = static_cast<uint32_t>(halo_bytes);
       p.g_stride = static_cast<uint32_t>(stage_g);
-      finish(2 * halo_bytes, depth * stage_g, 2);
+      finish(hbufs * halo_bytes, depth * stage_g, hbufs);
       return true;
     }
     const size_t tile_bytes = static_cast<size_t>(bmt) * p.row_bytes;
@@ -435,7 +451,7 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
       p.NBc >= period_ch && p.smem_bytes + round_up(kEpiStageBytes, 16) <= kBudget) {
     p.e_stage = 1;
     p.off_bar = static_cast<uint32_t>(round_up(p.off_e + kEpiStageBytes, 16));
-    p.smem_bytes = 1024 + p.off_bar + bar_bytes(p.stages, p.halo ? 2 : p.stages_a);
+    p.smem_bytes = 1024 + p.off_bar + bar_bytes(p.stages, p.halo ? p.hbufs : p.stages_a);
   }
   // Fused 2x2 max-pool (placed above): even output sizes, outputs of 1, 2, 4
   // or 8 bits in 32-bit words. A tile is q = 128 hv / (2 Wp) row pairs of
@@ -464,7 +480,7 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
     size_t off_e = 0;
     for (; depth >= 2; --depth) {
       off_e = round_up(p.off_g + static_cast<size_t>(depth) * p.g_stride, 16);
-      if (1024 + round_up(off_e + pool_bytes, 16) + bar_bytes(p.stages, 2) <= kBudget) break;
+      if (1024 + round_up(off_e + pool_bytes, 16) + bar_bytes(p.stages, p.hbufs) <= kBudget) break;
     }
     if (depth < 2) return SAMD_EUNSUP;
     p.pool = 1;
@@ -472,7 +488,7 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
     p.grid_m = static_cast<long long>(d->N) * p.pool_tpi;
     p.off_e = static_cast<uint32_t>(off_e);
     p.off_bar = static_cast<uint32_t>(round_up(off_e + pool_bytes, 16));
-    p.smem_bytes = 1024 + p.off_bar + bar_bytes(p.stages, 2);
+    p.smem_bytes = 1024 + p.off_bar + bar_bytes(p.stages, p.hbufs);
   }
   uint32_t cols = 32;
   while (cols < static_cast<uint32_t>(2 * p.hv * p.mma_n)) cols <<= 1;  // two accumulators of hv halves
@@ -486,14 +502,14 @@ samd_fmt none_fmt() { return samd_fmt{0, 0, 0, 0}; }
 // Every shared-memory region of the plan lies inside its allocation (checked
 // before each launch; a planning mistake becomes SAMD_EUNSUP, not a fault).
 bool layout_ok(const Plan &p) {
-  const size_t NO = p.halo ? 2 : static_cast<size_t>(p.stages_a);
+  const size_t NO = p.halo ? static_cast<size_t>(p.hbufs) : static_cast<size_t>(p.stages_a);
   const size_t op_bytes = NO * p.op_stride;
   const size_t bars = (2 * static_cast<size_t>(p.stages) + 2 * NO + 7) * 8 + 4;
   return p.stages >= 1 && NO >= 2 && op_bytes <= p.off_b &&
          p.off_b + static_cast<size_t>(p.stages) * p.b_bytes <= p.off_g && p.off_g + static_cast<size_t>(p.halo ? p.gdepth : 2) * p.g_stride <= p.off_e &&
          p.off_e <= p.off_bar && 1023 + p.off_bar + bars <= p.smem_bytes && p.op_stride % 1024 == 0 &&
          p.off_b % 1024 == 0 && p.b_bytes % 1024 == 0 && p.off_bar % 8 == 0 && 2 * p.hv * p.mma_n <= 512 &&
-         (p.hv == 1 || p.hv == 2) && (!p.halo || (p.gdepth >= 2 && p.gdepth <= 4)) &&
+         (p.hv == 1 || p.hv == 2) && (!p.halo || (p.gdepth >= 2 && p.gdepth <= 4 && (p.hbufs == 2 || p.hbufs == 3))) &&
          (!p.e_stage || p.off_e + kEpiStageBytes <= p.off_bar) &&
          (!p.pool || (p.halo && 2 * p.Wp <= BM * p.hv && !p.e_stage && p.pool_pitch >= p.pool_nw &&
                       p.off_e + static_cast<size_t>(2 * BM) * p.pool_pitch * 4 <= p.off_bar));
@@ -726,6 +742,7 @@ samd_status conv2d_run(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, const 
   a.off_g = p.off_g;
   a.g_stride = p.g_stride;
   a.gdepth = p.gdepth;
+  a.hbufs = p.hbufs;
   a.off_e = p.off_e;
   a.e_stage = p.e_stage;
   a.pool = p.pool;

@@ -162,6 +162,7 @@ struct ConvArgs {
   int gather_win;   // AGather::issue_win (chunks that are not aligned 16-byte vectors); chunk = (channel chunk, tap)
   int g_row;        // GATHER staging row pitch in bytes
   int gdepth;       // HALO: packed staging slots; gathers run gdepth - 1 items ahead
+  int hbufs;        // HALO: widened halo buffers (2 or 3); item k goes to buffer k mod hbufs
   long long act_bytes;  // bytes of the activation tensor (the windows stop at its end)
   uint32_t tmem_cols;
   int out_bits, out_signed, out_lane_w, out_L, out_word64, out_wpr;
@@ -1164,7 +1165,7 @@ __device__ __forceinline__ void issue_taps(uint32_t d, uint32_t dn, uint64_t a, 
 //   warps 2-9   operand producers.
 //               HALO: for each (tile, channel chunk) the halo rows the tile
 //               needs are gathered with cp.async and widened once into one of
-//               two halo buffers; every tap reads the halo through a
+//               two or three halo buffers; every tap reads the halo through a
 //               descriptor shifted by r * row_step + s rows.
 //               GATHER: each thread gathers its pixel's packed words (implicit
 //               im2col, zero padding) through a cp.async ring and widens them
@@ -1194,12 +1195,12 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
   const int STB = args.stages;  // weight tiles in flight (or resident)
   const bool resident = args.b_resident != 0;
   const uint32_t b_bytes = args.b_bytes;
-  uint8_t *sOp = smem;  // HALO: 2 halo buffers; GATHER: stages_a A tiles
+  uint8_t *sOp = smem;  // HALO: hbufs halo buffers; GATHER: stages_a A tiles
   uint8_t *sB = smem + args.off_b;
   uint8_t *sG = smem + args.off_g;  // packed staging
   uint64_t *bars = reinterpret_cast<uint64_t *>(smem + args.off_bar);
   // barriers: full_b[STB] empty_b[STB] opfull[NO] opempty[NO] accfull[2] accempty[2] drain group[2]
-  const int NO = HALO ? 2 : args.stages_a;
+  const int NO = HALO ? args.hbufs : args.stages_a;
   uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + 2 * STB + 2 * NO + 7);
   auto full_b = [&](int s) { return ptx::smem_addr(bars + s); };
   auto empty_b = [&](int s) { return ptx::smem_addr(bars + STB + s); };
@@ -1471,8 +1472,8 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
           ptx::cp_async_wait<2>();
         else
           ptx::cp_async_wait<1>();  // item k of this thread's rows has landed
-        const int hb = static_cast<int>(k & 1);
-        if (k >= 2 && !wait_lane0(opempty(hb), static_cast<uint32_t>(((k >> 1) - 1) & 1))) {
+        const int hb = static_cast<int>(k % NO);
+        if (k >= NO && !wait_lane0(opempty(hb), static_cast<uint32_t>(((k / NO) - 1) & 1))) {
           ok = false;
           break;
         }
