@@ -414,15 +414,25 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
     }
     return false;
   };
-  // Preference: resident weights, then halo over gather, then two-half tiles
-  // (two accumulators of 2 * mma_n TMEM columns each: mma_n <= 128).
+  // Preference: resident weights, then halo over gather, then the most
+  // 128-row parts per tile: four (e4m3 halo layers with at most 64 MMA
+  // columns: two accumulators of 4 x 64 TMEM columns), two (mma_n <= 128),
+  // one. A tile pays a fixed cost (its operand and accumulator handshakes,
+  // about 0.7 us measured) whatever its MMA count, so larger tiles of small-N
+  // layers spend more of their time in the MMAs -- when every SM gets many
+  // of them: four-part tiles are taken for layers of at least four per SM
+  // (VGG-16 conv2: 530 -> 622 TMAC/s); small layers, whose CTAs run a few
+  // tiles after a start-up of about 3 us, measured no gain or a loss.
   const bool two = p.mma_n <= 128;
+  const long long virt = static_cast<long long>(d->N) * (d->H + 2 * d->pad) * (d->W + 2 * d->pad);
+  const bool four = p.fp8 && p.mma_n <= 64 && (virt + 4 * BM - 1) / (4 * BM) >= 4LL * sm_count();
   bool placed = false;
+  const int kModes[5][2] = {{1, 4}, {1, 2}, {1, 1}, {0, 2}, {0, 1}};  // (halo, parts)
   for (int need_res = (p.nblocks == 1 ? 1 : 0); need_res >= 0 && !placed; --need_res)
-    for (int mode = 0; mode < 4 && !placed; ++mode) {
-      const bool halo = mode < 2;
-      const int hv = (mode % 2 == 0) ? 2 : 1;
-      if (hv == 2 && !two) continue;
+    for (int mode = 0; mode < 5 && !placed; ++mode) {
+      const bool halo = kModes[mode][0] != 0;
+      const int hv = kModes[mode][1];
+      if ((hv == 2 && !two) || (hv == 4 && !four)) continue;
       placed = place(halo, hv, need_res != 0);
     }
   if (!placed) return SAMD_EUNSUP;  // operand tiles do not fit (not reached for N <= 256)
@@ -509,7 +519,7 @@ bool layout_ok(const Plan &p) {
          p.off_b + static_cast<size_t>(p.stages) * p.b_bytes <= p.off_g && p.off_g + static_cast<size_t>(p.halo ? p.gdepth : 2) * p.g_stride <= p.off_e &&
          p.off_e <= p.off_bar && 1023 + p.off_bar + bars <= p.smem_bytes && p.op_stride % 1024 == 0 &&
          p.off_b % 1024 == 0 && p.b_bytes % 1024 == 0 && p.off_bar % 8 == 0 && 2 * p.hv * p.mma_n <= 512 &&
-         (p.hv == 1 || p.hv == 2) && (!p.halo || (p.gdepth >= 2 && p.gdepth <= 4 && (p.hbufs == 2 || p.hbufs == 3))) &&
+         (p.hv == 1 || p.hv == 2 || (p.hv == 4 && p.halo && p.fp8 && p.mma_n <= 64)) && (!p.halo || (p.gdepth >= 2 && p.gdepth <= 4 && (p.hbufs == 2 || p.hbufs == 3))) &&
          (!p.e_stage || p.off_e + kEpiStageBytes <= p.off_bar) &&
          (!p.pool || (p.halo && 2 * p.Wp <= BM * p.hv && !p.e_stage && p.pool_pitch >= p.pool_nw &&
                       p.off_e + static_cast<size_t>(2 * BM) * p.pool_pitch * 4 <= p.off_bar));

@@ -1092,13 +1092,18 @@ __device__ __forceinline__ void mma_op(uint32_t d, uint64_t a, uint64_t b, uint3
     ptx::mma_f16(d, a, b, idesc, acc);
 }
 
-// For a tile of HV halves of 128 rows, each k-step issues one MMA per half:
-// half h accumulates into d + h * dn from A rows 128 h on (a + h * ah).
+// For a tile of HV parts of 128 rows (HV = 1, 2, 4), each k-step issues one
+// MMA per part: part h accumulates into d + h * dn from A rows 128 h on
+// (a + h * ah).
 template <bool FP8, int HV>
 __device__ __forceinline__ void mma_kstep(uint32_t d, uint32_t dn, uint64_t a, uint64_t ah, uint64_t b, uint32_t idesc,
                                           uint32_t acc) {
   mma_op<FP8>(d, a, b, idesc, acc);
-  if constexpr (HV == 2) mma_op<FP8>(d + dn, a + ah, b, idesc, acc);
+  if constexpr (HV >= 2) mma_op<FP8>(d + dn, a + ah, b, idesc, acc);
+  if constexpr (HV == 4) {
+    mma_op<FP8>(d + 2 * dn, a + 2 * ah, b, idesc, acc);
+    mma_op<FP8>(d + 3 * dn, a + 3 * ah, b, idesc, acc);
+  }
 }
 
 // Issues `ksteps` (1..4) k-steps of one operand row as straight-line code.
@@ -1232,10 +1237,10 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     }
     for (int a = 0; a < 2; ++a) {
       ptx::mbar_init(accfull(a), 1);
-      ptx::mbar_init(accempty(a), HV == 2 ? kEpiWarps : kEpiWarps / 2);  // the warps that drain accumulator a
+      ptx::mbar_init(accempty(a), HV >= 2 ? kEpiWarps : kEpiWarps / 2);  // the warps that drain accumulator a
     }
     ptx::mbar_init(drain_bar, 1);
-    for (int g = 0; g < 2; ++g) ptx::mbar_init(group_bar(g), HV == 2 ? kEpiWarps : kEpiWarps / 2);
+    for (int g = 0; g < 2; ++g) ptx::mbar_init(group_bar(g), HV >= 2 ? kEpiWarps : kEpiWarps / 2);
     ptx::fence_barrier_init();
   }
   __syncwarp();  // every warp reaches the barrier converged (bar.sync counts whole warps)
@@ -1595,8 +1600,12 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         args.e_stage ? reinterpret_cast<uint32_t *>(smem + args.off_e) + (warp - kFirstEpiWarp) * 32 * kEpiPitch
                      : nullptr;
     const int row = quad * 32 + lane;
-    constexpr int kTileStep = HV == 2 ? 1 : 2;
-    long long i = HV == 2 ? 0 : set;
+    constexpr int kTileStep = HV >= 2 ? 1 : 2;
+    // parts of 128 rows of a tile this warp drains: set `set` takes parts
+    // set * kParts .. set * kParts + kParts - 1 (HV = 2: its half; HV = 4:
+    // two of the four parts); with HV = 1 the sets take alternate tiles
+    constexpr int kParts = HV == 4 ? 2 : 1;
+    long long i = HV >= 2 ? 0 : set;
     // The first pass over the first tile runs with its stores off and without
     // waiting for the accumulator (whatever it reads is discarded): the row
     // epilogue is the largest code of the kernel, and this way its
@@ -1604,7 +1613,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     // than after it.
     bool warm = true;
     bool pooled = false;
-    if constexpr (HALO) {
+    if constexpr (HALO && HV <= 2) {
       if (args.pool) {
         // pooled tiles (no warm-up pass): two-half tiles are drained and
         // pooled by all eight epilogue warps, one-half tiles by the four of
@@ -1641,8 +1650,8 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
         }
       }
     }
-    for (long long tile = first_tile + (HV == 2 ? 0 : set) * tile_step; !pooled && tile < total_tiles;) {
-      const int acc_i = HV == 2 ? static_cast<int>(i & 1) : set;  // accumulator of this tile
+    for (long long tile = first_tile + (HV >= 2 ? 0 : set) * tile_step; !pooled && tile < total_tiles;) {
+      const int acc_i = HV >= 2 ? static_cast<int>(i & 1) : set;  // accumulator of this tile
       if (!warm) {
         bool w_ok = true;
         if (lane == 0)
@@ -1657,24 +1666,28 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
       const uint32_t nbu = fdiv(tl, args.fd_gm);
       const int nb = static_cast<int>(nbu);
       const uint32_t mt = tl - nbu * args.fd_gm.d;
-      bool valid;
-      long long m;
-      const int trow = (HV == 2 ? set * BM : 0) + row;  // row of the tile
-      if (HALO) {
-        const uint32_t v = tile_first_pos(args, mt, BMT) + trow;
-        const uint32_t img = fdiv(v, args.fd_plane);
-        const uint32_t rem = v - img * args.fd_plane.d;
-        const uint32_t oh = fdiv(rem, args.fd_wp);
-        const uint32_t ow = rem - oh * args.fd_wp.d;
-        valid = static_cast<int>(img) < args.N && static_cast<int>(oh) < args.Ho && static_cast<int>(ow) < args.Wo;
-        m = (static_cast<long long>(img) * args.Ho + oh) * args.Wo + ow;
-      } else {
-        m = static_cast<long long>(mt) * BMT + trow;
-        valid = m < args.M;
+#pragma unroll 1
+      for (int hh = 0; hh < kParts; ++hh) {
+        const int part = HV >= 2 ? set * kParts + hh : 0;
+        bool valid;
+        long long m;
+        const int trow = part * BM + row;  // row of the tile
+        if (HALO) {
+          const uint32_t v = tile_first_pos(args, mt, BMT) + trow;
+          const uint32_t img = fdiv(v, args.fd_plane);
+          const uint32_t rem = v - img * args.fd_plane.d;
+          const uint32_t oh = fdiv(rem, args.fd_wp);
+          const uint32_t ow = rem - oh * args.fd_wp.d;
+          valid = static_cast<int>(img) < args.N && static_cast<int>(oh) < args.Ho && static_cast<int>(ow) < args.Wo;
+          m = (static_cast<long long>(img) * args.Ho + oh) * args.Wo + ow;
+        } else {
+          m = static_cast<long long>(mt) * BMT + trow;
+          valid = m < args.M;
+        }
+        const uint32_t taddr = tmem_base + static_cast<uint32_t>((acc_i * HV + part) * args.mma_n) +
+                               (static_cast<uint32_t>(quad * 32) << 16);
+        epilogue_row(args, taddr, valid && !warm, m, nb, estage);
       }
-      const uint32_t taddr = tmem_base + static_cast<uint32_t>((acc_i * HV + (HV == 2 ? set : 0)) * args.mma_n) +
-                             (static_cast<uint32_t>(quad * 32) << 16);
-      epilogue_row(args, taddr, valid && !warm, m, nb, estage);
       if (warm) {
         warm = false;
         continue;
@@ -1718,6 +1731,17 @@ cudaError_t launch_conv(const CUtensorMap &tmap, const ConvArgs &args, bool halo
       kern = halo ? conv_kernel<W, BITS, SIGNED, true, FP8, true, 2> : conv_kernel<W, BITS, SIGNED, false, FP8, true, 2>;
     else if (args.full)
       kern = halo ? conv_kernel<W, BITS, SIGNED, true, FP8, true, 1> : conv_kernel<W, BITS, SIGNED, false, FP8, true, 1>;
+  }
+  // four-part tiles: halo layers on e4m3 operands only (planned so)
+  if constexpr (FP8) {
+    if (args.hv == 4) {
+      if (!halo) return cudaErrorInvalidValue;
+      kern = conv_kernel<W, BITS, SIGNED, true, FP8, false, 4>;
+      if constexpr (kHasFull)
+        if (args.full) kern = conv_kernel<W, BITS, SIGNED, true, FP8, true, 4>;
+    }
+  } else {
+    if (args.hv == 4) return cudaErrorInvalidValue;
   }
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void *>(kern), smem);
   if (e != cudaSuccess) return e;

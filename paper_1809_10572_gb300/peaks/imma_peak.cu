@@ -39,7 +39,7 @@ __global__ void __launch_bounds__(256) imma_loop_kernel(int iters, int seed, int
   if (s == 0x12345678) out[0] = s;  // keeps the results live; practically never taken
 }
 
-// The binary path SURVEY names for 1-2-bit lanes: mma.sync m16n8k256 on b1
+// A binary path for 1-2-bit lanes: mma.sync m16n8k256 on b1
 // operands with AND + popcount accumulation into s32 (a 1-bit x 1-bit
 // product per bit pair). A b-bit x b-bit multiply-add built from bit planes
 // takes b^2 of these products, so this rate bounds such a convolution.

@@ -37,7 +37,7 @@ samd_status conv2d_nchw(const samd_conv_desc *, samd_fmt, const void *, samd_fmt
 
 int main() {
   using namespace samd;
-  long long n = 0, bad = 0, halo = 0, seg = 0, fp8 = 0, res = 0, unsup = 0, hv2 = 0, win = 0, deep = 0, estg = 0;
+  long long n = 0, bad = 0, halo = 0, seg = 0, fp8 = 0, res = 0, unsup = 0, hv2 = 0, win = 0, deep = 0, estg = 0, hv4 = 0;
   const int Cs[] = {1, 3, 16, 24, 64, 96, 128, 256, 512, 1024};
   const int Ks[] = {1, 16, 40, 64, 96, 128, 256, 300, 512, 1024};
   const int HWs[] = {1, 2, 7, 14, 28, 56, 224};
@@ -52,7 +52,7 @@ int main() {
                   for (int rs : {1, 3, 5})
                     for (int st : {1, 2}) {
                       if (rs > hw + 2) continue;
-                      samd_conv_desc d{2, C, hw, hw, K, rs, rs, st, rs / 2, SAMD_NHWC};
+                      samd_conv_desc d{hw >= 112 ? 16 : 2, C, hw, hw, K, rs, rs, st, rs / 2, SAMD_NHWC};  // batch 16 for large images (four-part tiles)
                       samd_fmt fa{(uint8_t)ba, (uint8_t)sa, 0, (uint8_t)wb};
                       samd_fmt fw{(uint8_t)bw, (uint8_t)sw, 0, (uint8_t)wb};
                       for (int fob : {0, 3, 4, 6}) {
@@ -92,6 +92,7 @@ int main() {
                         if (p.fp8) ++fp8;
                         if (p.b_resident) ++res;
                         if (p.hv == 2) ++hv2;
+                        if (p.hv == 4) ++hv4;
                         ok = ok && p.tmem_cols <= 512 && 2 * p.hv * p.mma_n <= static_cast<int>(p.tmem_cols);
                         if (p.e_stage) {
                           ++estg;
@@ -103,7 +104,7 @@ int main() {
                       }
                     }
   printf("plans %lld, bad %lld, unsupported %lld, halo %lld (segmented %lld), e4m3 %lld, resident %lld, "
-         "two-half %lld, window gather %lld, staging at the chosen depth %lld, staged epilogue %lld\n",
-         n, bad, unsup, halo, seg, fp8, res, hv2, win, deep, estg);
+         "two-half %lld, four-part %lld, window gather %lld, staging at the chosen depth %lld, staged epilogue %lld\n",
+         n, bad, unsup, halo, seg, fp8, res, hv2, hv4, win, deep, estg);
   return bad != 0;
 }

@@ -28,7 +28,7 @@ def test_every_plan_fits_and_does_not_overlap():
         assert r.returncode == 0, r.stdout[-2000:]
         assert "bad 0" in r.stdout
         # the grid reaches every planning mode
-        for mode in ("halo", "segmented", "e4m3", "resident", "two-half", "window gather", "staging at the chosen depth",
+        for mode in ("halo", "segmented", "e4m3", "resident", "two-half", "four-part", "window gather", "staging at the chosen depth",
                      "staged epilogue"):
             count = int(r.stdout.split(mode)[1].split()[0].strip("(),"))
             assert count > 0, (mode, r.stdout)
