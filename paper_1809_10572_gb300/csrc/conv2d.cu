@@ -250,6 +250,10 @@ samd_status make_plan(const samd_conv_desc *d, samd_fmt fa, samd_fmt fw, samd_fm
   p.M = static_cast<long long>(d->N) * p.Ho * p.Wo;
   // A channel block must cover whole output words so that no packed word is
   // shared by two CTAs.
+  // Channel blocks of up to 256 MMA columns (128 with split digits). (Blocks
+  // of 128 for layers with few output positions, which doubles their CTAs,
+  // measured slower: every block gathers and widens the whole A operand
+  // again, and those layers are bound by that work.)
   const int limit = p.split ? 128 : 256;
   if (d->K <= limit) {
     p.NBc = d->K;

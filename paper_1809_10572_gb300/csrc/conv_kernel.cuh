@@ -180,7 +180,7 @@ struct ConvArgs {
   int nseg, seg_rows, seg_used, row_step;
   int nck;   // channel chunks per pixel (ceil(wpr / WC))
   int full;  // AUnpack FULL: one chunk holds all the pixel's words
-  int hv;    // tile of hv halves of 128 output positions (1 or 2)
+  int hv;    // tile of hv parts of 128 output positions (1, 2, or 4 for e4m3 halo layers)
   int taps;  // R * S
   FastDiv fd_plane, fd_wp;  // / (Hv * Wp), / Wp
   FastDiv fd_seg;           // / seg_rows
@@ -1158,9 +1158,9 @@ __device__ __forceinline__ void issue_taps(uint32_t d, uint32_t dn, uint64_t a, 
 //
 // One CTA per SM loops over output tiles (tile = blockIdx.x + i * gridDim.x;
 // tile = nb * grid_m + mt: channel block nb, position tile mt of 128 * HV
-// positions; HV = 2 issues each k-step's MMA for both 128-row halves and
-// halves the synchronization per MMA). Eighteen
-// warps with fixed roles, connected by mbarrier rings:
+// positions; with HV = 2 or 4 each k-step issues one MMA per 128-row part,
+// so the parts share every synchronization). Eighteen warps with fixed
+// roles, connected by mbarrier rings:
 //   warp 0      TMEM allocation; lane 0 streams weight tiles with TMA. When
 //               the layer has one channel block and all its weight tiles fit,
 //               they are loaded once and stay resident.
@@ -1176,15 +1176,18 @@ __device__ __forceinline__ void issue_taps(uint32_t d, uint32_t dn, uint64_t a, 
 //               im2col, zero padding) through a cp.async ring and widens them
 //               into a ring of A tiles; with HV = 1 two groups of four warps
 //               take alternate (tile, chunk) items, with HV = 2 the two groups
-//               fill the two halves of every item. 1x1 layers whose pixel
-//               rows are not 16-byte multiples copy 16-byte windows.
+//               fill the two halves of every item. Chunks that are not whole
+//               16-byte vectors are copied as 16-byte windows.
 //   warps 10-17 epilogue: tcgen05.ld, exact integers, optional int32 store,
 //               optional requantize-and-pack. HV = 1: warps 10-13 drain
 //               accumulator 0 (the CTA's even tiles), warps 14-17
 //               accumulator 1; HV = 2: warps 10-13 drain the first half and
-//               14-17 the second half of every tile. Warp w reads the TMEM
-//               lanes of quadrant w % 4. A first, store-free pass over the
-//               first tile fetches the epilogue's code early.
+//               14-17 the second half of every tile; HV = 4 (halo layers on
+//               e4m3 operands): warps 10-13 drain parts 0 and 1, 14-17 parts
+//               2 and 3. Warp w reads the TMEM lanes of quadrant w % 4. A
+//               first, store-free pass over the first tile fetches the
+//               epilogue's code early. Pooled tiles (ConvArgs::pool) are
+//               drained, requantized and pooled by the warps of a group.
 // Every wait is bounded; a role that gives up records SAMD_ETIMEOUT and stops.
 template <typename W, int BITS, bool SIGNED, bool HALO, bool FP8, bool FULL, int HV>
 __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant__ CUtensorMap tmap_b,
@@ -1309,7 +1312,7 @@ __global__ void __launch_bounds__(kThreads, 1) conv_kernel(const __grid_constant
     const int nops = HALO ? args.nck : nchunks;  // operand stages per tile
     const int taps_here = HALO ? args.taps : 1;
     constexpr uint32_t a_row16 = T::kRowBytes / 16;  // one operand row in descriptor units
-    constexpr uint64_t a_half16 = static_cast<uint64_t>(BM) * a_row16;  // the second half's first A row
+    constexpr uint64_t a_half16 = static_cast<uint64_t>(BM) * a_row16;  // from one 128-row part's A rows to the next
     const uint32_t dn = static_cast<uint32_t>(args.mma_n);          // the second half's accumulator columns
     const uint32_t a_skip16 = HALO ? static_cast<uint32_t>(args.row_step - args.S) * a_row16 : 0u;
     if (resident)  // resident weights: wait for all of them once
