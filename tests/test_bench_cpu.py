@@ -36,3 +36,24 @@ def test_traffic_reported_only_while_sources_match(bench, monkeypatch):
     assert value is None and "changed" in note
     for args in (types.SimpleNamespace(workload="vgg16", layers=""), types.SimpleNamespace(workload="sweep", layers="12")):
         assert bench.measured_traffic(args)[0] is None
+
+
+def test_chained_step_bookkeeping(bench):
+    """A chained network shares buffers between layers: each distinct tensor
+    counts once toward the bytes that decide how many input sets rotate, and
+    a layer whose pool is fused is one launch, a standalone pool a second."""
+    import torch
+
+    def t(n):
+        return torch.empty(n, dtype=torch.int32)
+
+    a0, o0, p0, o1, o2 = t(100), t(50), t(10), t(40), t(20)
+    conv = lambda n: types.SimpleNamespace(prepared=t(n))
+    built = [
+        {"act": a0, "out": o0, "conv": conv(8), "pooled": p0, "fused_pool": False},  # conv, then a pool launch
+        {"act": p0, "out": o1, "conv": conv(8), "pooled": None, "fused_pool": False},
+        {"act": o1, "out": o2, "conv": conv(8), "pooled": t(5), "fused_pool": True},  # pool in the epilogue
+    ]
+    assert bench.launches_per_step(built) == 4
+    want = 4 * (100 + 50 + 10 + 40 + 20 + 5 + 3 * 8)  # p0 and o1 counted once
+    assert bench.unique_bytes(built) == want
