@@ -44,6 +44,10 @@ def parse_args():
     ap.add_argument("--impl", default="samd", choices=["samd", "reference"])
     ap.add_argument("--workload", default="sweep", choices=["sweep", "vgg16", "resnet50", "conv1x"])
     ap.add_argument("--no-packed-ops", action="store_true")
+    ap.add_argument("--profile-fused-pool", action="store_true",
+                    help="VGG-16 conv7 (N16 C256->256 56x56, u4 x s4 -> u4) with the 2x2 max-pool fused into its "
+                         "epilogue, one untimed call and one more, and exit: the command ncu captures for the fused "
+                         "pool")
     ap.add_argument("--profile-ops", action="store_true",
                     help="launch each packed op once at 2^28 lanes (b = 1, 4, 8; pack, unpack, the five elementwise "
                          "ops) and the VGG-16 block-1 max-pool, after one untimed warm-up launch of each, and exit: "
@@ -523,6 +527,31 @@ def profile_ops():
     return 0
 
 
+def profile_fused_pool():
+    """VGG-16 conv7 with its pool fused (samd_conv2d_prepared_pool2x2): the
+    first call is a warm-up, the second the one profiled (ncu -s 1 -c 1)."""
+    import torch
+
+    from paper_1809_10572_gb300 import samd, synth, workloads
+
+    dev = torch.device("cuda", 0)
+    samd.load()
+    layer = next(l for l in workloads.vgg16() if l.name == "conv7")
+    s = layer.shape
+    fa, fw, fo = samd.fmt(layer.ba, layer.sa), samd.fmt(layer.bw, layer.sw), samd.fmt(layer.bo, layer.so)
+    a_w = samd.pack(synth.to_bytes_t(synth.lanes_t(11, (s.N * s.H * s.W, s.C), layer.ba, layer.sa, device=dev)), fa)
+    w_w = samd.pack(synth.to_bytes_t(synth.lanes_t(12, (s.K * s.R * s.S, s.C), layer.bw, layer.sw, device=dev)), fw)
+    conv = samd.PreparedConv(w_w, s, fa, fw, fo)
+    pooled = samd.empty_words(fo, s.N * (s.Ho // 2) * (s.Wo // 2), s.K, dev)
+    shift = workloads.harness_shift(layer.ba, layer.bw, layer.bo, s.C * s.R * s.S)
+    for _ in range(2):
+        conv.pool2x2(a_w, pooled, shift)
+    torch.cuda.synchronize()
+    print(json.dumps({"profile_fused_pool": layer.name, "pooled_bytes": pooled.numel() * 4,
+                      "input_bytes": a_w.numel() * 4}), flush=True)
+    return 0
+
+
 def csrc_digest():
     """sha256 over the kernel sources (file names and contents)."""
     h = hashlib.sha256()
@@ -968,6 +997,8 @@ def main():
 
     if args.profile_ops:
         return profile_ops()
+    if args.profile_fused_pool:
+        return profile_fused_pool()
     layers = workloads.WORKLOADS[args.workload]()
     if args.layers:
         idx = [int(t) for t in args.layers.split(",")]
