@@ -112,11 +112,30 @@ __device__ __forceinline__ W swar_mul(W a, W b) {
   return acc;
 }
 
+// Wrapping lane product on the integer multiplier without taking a's lane
+// out: with s the lane's offset and M = (2^bits - 1) << s its data bits,
+// b & M is b_i * 2^s, so (a >> s) * (b & M) = ((a >> s) * b_i) << s, whose
+// bits [s, s + bits) are a_i * b_i mod 2^bits (the bits of a above lane i
+// reach only higher product bits). One shift, one multiply and two logic
+// operations per lane; the low bits are the same for signed and unsigned
+// lanes (section 4.1). 32-bit words only (s + bits <= 32).
+__device__ __forceinline__ uint32_t lane_mul_at(uint32_t r, uint32_t a, uint32_t b, int s, uint32_t M) {
+  return r | (((a >> s) * (b & M)) & M);
+}
+
 // Lane-by-lane multiply (cheaper than shift-and-add from 3-bit lanes up).
 template <typename W, int BITS>
 __device__ __forceinline__ W lane_mul(W a, W b, bool is_signed, bool sat) {
   constexpr int L = Masks<W, BITS>::L;
   constexpr uint32_t LM = (1u << BITS) - 1;
+  if constexpr (sizeof(W) == 4) {
+    if (!sat) {
+      uint32_t r = 0;
+#pragma unroll
+      for (int i = 0; i < L; ++i) r = lane_mul_at(r, a, b, i * BITS, LM << (i * BITS));
+      return r;
+    }
+  }
   const int lo = lane_lo(BITS, is_signed), hi = lane_hi(BITS, is_signed);
   W r = 0;
 #pragma unroll
@@ -327,7 +346,8 @@ __device__ __forceinline__ W field_mul(W a, W b, const FieldMasks<W> &f, bool is
     // steps of a few word operations each, against L lanes of extract,
     // multiply and insert (measured: shift-and-add wins while bits <= L,
     // e.g. 0.51 -> 0.90 of HBM at 3-bit lanes with one spacer bit in 32-bit
-    // words, and loses at 6 and 7 bits, four lanes per word)
+    // words, and loses at 6 and 7 bits, four lanes per word). 32-bit words
+    // reach this only where field_mul_by_lanes declines the multiplier form.
     W acc = 0;
     for (int j = 0; j < f.bits; ++j) {
       const W bit = b & (f.lsb << j);
@@ -353,6 +373,28 @@ __device__ __forceinline__ W field_mul(W a, W b, const FieldMasks<W> &f, bool is
   return r;
 }
 
+// The wrapping multiply of V words of 32-bit spacer-separated fields, lane
+// outermost so the runtime lane loop's bookkeeping is shared by the words
+// (lane_mul_at per field).
+template <int V>
+__device__ __forceinline__ void field_mul_lanes(const uint32_t *a, const uint32_t *b, uint32_t *o,
+                                                const FieldMasks<uint32_t> &f) {
+#pragma unroll
+  for (int k = 0; k < V; ++k) o[k] = 0;
+  uint32_t M = (1u << f.bits) - 1;
+  for (int s = 0, i = 0; i < f.L; ++i, s += f.fw, M <<= f.fw) {
+#pragma unroll
+    for (int k = 0; k < V; ++k) o[k] = lane_mul_at(o[k], a[k], b[k], s, M);
+  }
+}
+
+// Per word, shift-and-add costs about nine operations a step (bits steps)
+// and field_mul_lanes about five a lane (L lanes): take the lanes form where
+// it is cheaper (from 4-bit lanes with one spacer bit in 32-bit words).
+__device__ __forceinline__ bool field_mul_by_lanes(const FieldMasks<uint32_t> &f) {
+  return 5 * f.L < 9 * f.bits;
+}
+
 template <typename W, int OP>
 __device__ __forceinline__ W field_op(W a, W b, const FieldMasks<W> &f, bool is_signed, bool sat, int shift,
                                       W keep) {
@@ -363,8 +405,10 @@ __device__ __forceinline__ W field_op(W a, W b, const FieldMasks<W> &f, bool is_
   else return field_shift<W>(a, shift, keep, f, is_signed);
 }
 
+// Held to 8 CTAs of 256 threads per SM (32 registers): the multiply's two
+// forms in one kernel would otherwise take 40 and fit 6.
 template <typename W, int OP>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 8)
     ew_field_kernel(const W *__restrict__ a, const W *__restrict__ b, W *__restrict__ out, int64_t nwords,
                     const FieldMasks<W> f, int is_signed, int sat, int shift) {
   constexpr int V = 16 / sizeof(W);
@@ -384,8 +428,17 @@ __global__ void __launch_bounds__(kThreads)
     W wa[V], wb[V], wo[V];
     memcpy(wa, &ra, 16);
     memcpy(wb, &rb, 16);
+    if constexpr (OP == SAMD_MUL && sizeof(W) == 4) {
+      if (!sat && field_mul_by_lanes(f)) {
+        field_mul_lanes<V>(wa, wb, wo, f);
+      } else {
 #pragma unroll
-    for (int k = 0; k < V; ++k) wo[k] = field_op<W, OP>(wa[k], wb[k], f, is_signed, sat, shift, keep);
+        for (int k = 0; k < V; ++k) wo[k] = field_op<W, OP>(wa[k], wb[k], f, is_signed, sat, shift, keep);
+      }
+    } else {
+#pragma unroll
+      for (int k = 0; k < V; ++k) wo[k] = field_op<W, OP>(wa[k], wb[k], f, is_signed, sat, shift, keep);
+    }
     uint4 ro;
     memcpy(&ro, wo, 16);
     __stcs(reinterpret_cast<uint4 *>(out) + v, ro);
@@ -393,6 +446,14 @@ __global__ void __launch_bounds__(kThreads)
   for (int64_t w = nvec * V + blockIdx.x * (int64_t)blockDim.x + threadIdx.x; w < nwords; w += stride) {
     const W x = a[w];
     const W y = kBinary ? b[w] : x;
+    if constexpr (OP == SAMD_MUL && sizeof(W) == 4) {
+      if (!sat && field_mul_by_lanes(f)) {
+        uint32_t r;
+        field_mul_lanes<1>(&x, &y, &r, f);
+        out[w] = r;
+        continue;
+      }
+    }
     out[w] = field_op<W, OP>(x, y, f, is_signed, sat, shift, keep);
   }
 }
@@ -401,17 +462,23 @@ template <typename W>
 cudaError_t field_dispatch(samd_op op, samd_fmt f, const void *a, const void *b, void *out, int64_t n, int shift,
                            int sat, cudaStream_t s) {
   const int64_t nwords = words_per_row(f, n);
-  const int grid = grid_for(nwords / (16 / sizeof(W)) + 1, kThreads, sm_count() * 8);
+  const int64_t work = nwords / (16 / sizeof(W)) + 1;
   const FieldMasks<W> m = field_masks<W>(f);
   const W *pa = static_cast<const W *>(a);
   const W *pb = static_cast<const W *>(b);
   W *po = static_cast<W *>(out);
   switch (op) {
-    case SAMD_ADD: ew_field_kernel<W, SAMD_ADD><<<grid, kThreads, 0, s>>>(pa, pb, po, nwords, m, f.is_signed, sat, shift); break;
-    case SAMD_SUB: ew_field_kernel<W, SAMD_SUB><<<grid, kThreads, 0, s>>>(pa, pb, po, nwords, m, f.is_signed, sat, shift); break;
-    case SAMD_MUL: ew_field_kernel<W, SAMD_MUL><<<grid, kThreads, 0, s>>>(pa, pb, po, nwords, m, f.is_signed, sat, shift); break;
-    case SAMD_RELU: ew_field_kernel<W, SAMD_RELU><<<grid, kThreads, 0, s>>>(pa, pb, po, nwords, m, f.is_signed, sat, shift); break;
-    default: ew_field_kernel<W, SAMD_REQUANT><<<grid, kThreads, 0, s>>>(pa, pb, po, nwords, m, f.is_signed, sat, shift); break;
+#define SAMD_FIELD_CASE(OPC)                                                                     \
+  case OPC:                                                                                      \
+    ew_field_kernel<W, OPC><<<resident_grid<ew_field_kernel<W, OPC>>(work, kThreads), kThreads, 0, s>>>( \
+        pa, pb, po, nwords, m, f.is_signed, sat, shift);                                         \
+    break;
+    SAMD_FIELD_CASE(SAMD_ADD) SAMD_FIELD_CASE(SAMD_SUB) SAMD_FIELD_CASE(SAMD_MUL) SAMD_FIELD_CASE(SAMD_RELU)
+#undef SAMD_FIELD_CASE
+    default:
+      ew_field_kernel<W, SAMD_REQUANT><<<resident_grid<ew_field_kernel<W, SAMD_REQUANT>>(work, kThreads), kThreads,
+                                          0, s>>>(pa, pb, po, nwords, m, f.is_signed, sat, shift);
+      break;
   }
   return cudaGetLastError();
 }
@@ -420,14 +487,14 @@ template <typename W, int OP>
 cudaError_t swar_dispatch_bits(int bits, const void *a, const void *b, void *out, int64_t nwords, int is_signed,
                                int sat, int shift, cudaStream_t s) {
   int64_t work = nwords / Vec4<W>::kWords + 1;
-  int grid = grid_for(work, kThreads, sm_count() * 8);
   const W *pa = static_cast<const W *>(a);
   const W *pb = static_cast<const W *>(b);
   W *po = static_cast<W *>(out);
   switch (bits) {
 #define SAMD_EW_CASE(B) \
   case B:               \
-    ew_swar_kernel<W, B, OP><<<grid, kThreads, 0, s>>>(pa, pb, po, nwords, is_signed, sat, shift); \
+    ew_swar_kernel<W, B, OP><<<resident_grid<ew_swar_kernel<W, B, OP>>(work, kThreads), kThreads, 0, s>>>( \
+        pa, pb, po, nwords, is_signed, sat, shift);                                                    \
     break;
     SAMD_EW_CASE(1) SAMD_EW_CASE(2) SAMD_EW_CASE(3) SAMD_EW_CASE(4)
     SAMD_EW_CASE(5) SAMD_EW_CASE(6) SAMD_EW_CASE(7) SAMD_EW_CASE(8)

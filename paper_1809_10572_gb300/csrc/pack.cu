@@ -436,17 +436,18 @@ __global__ void __launch_bounds__(kThreads) unpack_generic_kernel(const W *__res
 
 template <int BITS>
 cudaError_t launch_pack32_vec(const int8_t *src, uint32_t *dst, int64_t ntiles, cudaStream_t s) {
-  const int grid = grid_for(ntiles * 32, kThreads, sm_count() * 8);
   if (BITS == 1)
-    pack32_staged_kernel<BITS><<<grid, kThreads, 0, s>>>(src, dst, ntiles);
+    pack32_staged_kernel<BITS><<<resident_grid<pack32_staged_kernel<BITS>>(ntiles * 32, kThreads), kThreads, 0, s>>>(
+        src, dst, ntiles);
   else
-    pack32_vec_kernel<BITS><<<grid, kThreads, 0, s>>>(src, dst, ntiles * 32);
+    pack32_vec_kernel<BITS><<<resident_grid<pack32_vec_kernel<BITS>>(ntiles * 32, kThreads), kThreads, 0, s>>>(
+        src, dst, ntiles * 32);
   return cudaGetLastError();
 }
 
 template <int BITS, bool SIGNED>
 cudaError_t launch_unpack32_vec(const uint32_t *src, int8_t *dst, int64_t ntiles, cudaStream_t s) {
-  const int grid = grid_for(ntiles * 32, kThreads, sm_count() * 8);
+  const int grid = resident_grid<unpack32_vec_kernel<BITS, SIGNED>>(ntiles * 32, kThreads);
   unpack32_vec_kernel<BITS, SIGNED><<<grid, kThreads, 0, s>>>(src, dst, ntiles);
   return cudaGetLastError();
 }

@@ -42,6 +42,31 @@ inline int grid_for(int64_t work_items, int threads, int max_blocks) {
 // Number of SMs of the current device (cached per device).
 int sm_count();
 
+// CTAs of `Kernel` resident on one SM at `threads` threads and `smem`
+// dynamic shared bytes (its registers and static shared memory decide), at
+// least 1; asked once per kernel.
+template <auto Kernel>
+int resident_ctas(int threads, size_t smem = 0) {
+  static const int n = [threads, smem] {
+    int r = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, Kernel, threads, smem) != cudaSuccess) {
+      (void)cudaGetLastError();  // the query's own error; the launch reports any other
+      r = 0;
+    }
+    return r < 1 ? 1 : r;
+  }();
+  return n;
+}
+
+// Grid of a grid-stride kernel: enough CTAs for the work, at most one full
+// wave of resident CTAs (sm_count() x resident_ctas). A grid of 8 CTAs per SM
+// for a kernel of which only 6 fit leaves a third of a wave to start late and
+// run its share on an emptier GPU.
+template <auto Kernel>
+int resident_grid(int64_t work_items, int threads, size_t smem = 0) {
+  return grid_for(work_items, threads, sm_count() * resident_ctas<Kernel>(threads, smem));
+}
+
 // ---- device-side lane helpers ----------------------------------------------
 
 template <typename W>

@@ -63,7 +63,7 @@ def test_elementwise_full_grid(samd_lib, bits, signed):
 
 
 @pytest.mark.parametrize("signed", (False, True))
-@pytest.mark.parametrize("bits", (1, 3, 7))
+@pytest.mark.parametrize("bits", (1, 3, 5, 7))
 def test_elementwise_full_grid_one_spacer_bit(samd_lib, bits, signed):
     # the permanent-spacer word forms (one zero bit above each lane, Fig. 2)
     f = samd.fmt(bits, signed, 1)

@@ -114,7 +114,8 @@ def test_requant_format_change(samd_lib, fa_t, fo_t):
 @pytest.mark.parametrize("op", ("add", "sub", "mul", "relu"))
 def test_ops_with_spacer_bits(samd_lib, op, spacer):
     for bits, signed, word_bits in [(3, True, 32), (4, False, 64), (7, True, 32), (1, False, 32), (2, True, 32),
-                                    (2, False, 64), (1, True, 32), (8, False, 64), (5, True, 64)]:
+                                    (2, False, 64), (1, True, 32), (8, False, 64), (5, True, 64), (4, True, 32),
+                                    (5, False, 32), (6, True, 32)]:
         f = samd.fmt(bits, signed, spacer, word_bits)
         n = 30011
         xv, xb = values_and_bytes(synth.seed_for("sx", op, bits, spacer), (n,), bits, signed)
