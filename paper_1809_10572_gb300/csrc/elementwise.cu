@@ -4,7 +4,8 @@
 // word-level (SAMD) forms: every lane of a word is updated by a handful of
 // whole-word integer instructions, the way section 3 of the paper adds and
 // subtracts with temporary spacer bits (Fig. 5) and multiplies by masked
-// shift-and-add (Fig. 6). On GB300 this keeps the per-word ALU cost below
+// shift-and-add (Fig. 6) at 1-2-bit lanes (from 3 bits, lane by lane on the
+// integer multiplier, lane_mul). On GB300 this keeps the per-word ALU cost below
 // what HBM bandwidth leaves per word even at 1-2 bit lanes, where a
 // lane-by-lane loop would run 16-32 iterations per word. Words move with
 // 128-bit loads and stores.
